@@ -1,0 +1,350 @@
+"""Benchmark: Ozaki Scheme II DGEMM emulation on FP8 tensor cores (GB300).
+
+One step = one full emulated DGEMM through the library's public entry point
+(oz2_dgemm: scan, "+1" pass, scales, deconstruction, residue GEMMs, Garner,
+fallback) on the seeded synthetic workload, inputs resident in HBM.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+                  [--num-moduli R] [--impl reference] [--no-sweep]
+
+Prints one JSON line (rank 0).  Under torchrun each rank runs an independent
+replica of the workload on its own GPU (the method needs no exchange for
+independent problems), and the value is the sum over ranks of the work
+divided by the slowest rank's time.
+
+--impl reference times the CPU oracle (oracle/) on the host cores on a
+bounded sample of the same workload and metric.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import workloads as wl  # noqa: E402
+
+METRIC = "effective FP64 TFLOPS (2mnk/s) and % of FP8 tensor peak/alpha, per moduli count"
+L2_BYTES = 126 * 2**20
+FP8_TO_BF16 = 2.0   # nominal dense FP8 / BF16 tensor ratio (4.5 / 2.25 PFLOP/s)
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=200)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--workload", default="dgemm_4096", choices=sorted(wl.WORKLOADS))
+    p.add_argument("--num-moduli", type=int, default=12)
+    p.add_argument("--impl", default="oz2", choices=["oz2", "reference"])
+    p.add_argument("--no-sweep", action="store_true")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    return p.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return {"hbm_gbs": d["hbm_gbs"], "bf16": d["bf16_tflops"], "bf16_sustained": d["bf16_tflops_sustained"],
+                "source": "measured"}
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16": 1900.0, "bf16_sustained": 1700.0, "source": "fallback"}
+
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling during the timed region."""
+
+    QUERY = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.QUERY}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        self.lines = [l for l in out.splitlines() if l.strip()]
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 10:
+                continue
+            try:
+                sm.append(float(f[2]))
+                mx = float(f[3])
+            except ValueError:
+                continue
+            for nm, v in zip(names, f[6:10]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def stage_bytes_flops(w, r, k_pad, P):
+    """Algorithmic work per stage (bytes moved or FP8 flops), per call."""
+    m, n, k = w.m, w.n, w.k
+    return {
+        "scan": ("hbm", 8.0 * (m * k + k * n)),
+        "magnitude": ("hbm", 8.0 * (m * k + k * n) + (m + n) * k_pad),
+        "plus_one_gemm": ("tensor", 2.0 * m * n * k_pad),
+        "deconstruct": ("hbm", 8.0 * (m * k + k * n) + P * (m + n) * k_pad),
+        "residue_gemm": ("tensor", 3.0 * r * 2.0 * m * n * k_pad),
+        "crt": ("hbm", 2.0 * r * m * n + 8.0 * m * n),
+    }
+
+
+def run_oz2(args):
+    import torch
+    import torch.distributed as dist
+
+    import paper_2606_06510_gb300 as oz
+    from oracle import cref
+
+    world, rank, local = dist_env()
+    if world > 1:
+        dist.init_process_group("gloo")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    w = wl.WORKLOADS[args.workload]
+    r = args.num_moduli
+    A, B = wl.make_inputs(w)
+    dA = oz.colmajor(torch.from_numpy(np.ascontiguousarray(A)).to(dev))
+    dB = oz.colmajor(torch.from_numpy(np.ascontiguousarray(B)).to(dev))
+    dC = torch.empty((w.n, w.m), dtype=torch.float64, device=dev).t()
+    stream = torch.cuda.current_stream()
+    in_bytes = 8 * (w.m * w.k + w.k * w.n)
+
+    def step():
+        oz.oz2_dgemm(dA, dB, C=dC, num_moduli=r)
+
+    # warm-up (also the first-use set-up of the plane table on this device)
+    for _ in range(max(args.warmup, 3)):
+        step()
+    torch.cuda.synchronize()
+    assert oz.oz2_check_device_status() == 0
+    oz.oz2_get_stats()                      # reset counters
+    flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device=dev)
+    flush.fill_(1.0)
+
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.3)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    sampler.stop()
+    ms = e0.elapsed_time(e1)
+    launches = oz.oz2_get_stats()["kernel_launches"]
+    assert oz.oz2_check_device_status() == 0
+    if world > 1:
+        t = torch.tensor([ms], dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    ms_per_step = ms / args.steps
+    value = world * w.flops / (ms_per_step * 1e-3) / 1e12
+
+    # Per-stage device times: the same steps with the library's stream events.
+    ws = torch.empty(oz.oz2_workspace_size(w.m, w.n, w.k, r), dtype=torch.uint8, device=dev)
+    nstage = min(args.steps, 50)
+    for _ in range(nstage):
+        oz.oz2_dgemm_ex(dA, dB, C=dC, num_moduli=r, flags=oz.FLAG_TIMING, workspace=ws)
+    st = oz.oz2_get_stats()
+    stage_ms = st["stage_ms"]
+    L = oz.oz2_workspace_layout(w.m, w.n, w.k, r)
+    work = stage_bytes_flops(w, r, L["k_pad"], L["num_planes"])
+    pk = peaks()
+    fp8_peak = pk["bf16_sustained"] * FP8_TO_BF16
+    stages = {}
+    for name, (kind, amount) in work.items():
+        t = stage_ms.get(name, 0.0)
+        if t <= 0:
+            continue
+        if kind == "hbm":
+            ach = amount / (t * 1e-3) / 1e9
+            stages[name] = {"ms": round(t, 4), "GB/s": round(ach, 1), "frac_hbm": round(ach / pk["hbm_gbs"], 3)}
+        else:
+            ach = amount / (t * 1e-3) / 1e12
+            stages[name] = {"ms": round(t, 4), "TFLOP/s_fp8": round(ach, 1), "frac_fp8": round(ach / fp8_peak, 3)}
+    gemm_ms = stage_ms["residue_gemm"]
+    gemm_flops = work["residue_gemm"][1]
+    achieved = gemm_flops / (gemm_ms * 1e-3) / 1e12
+    roofline = {"bound": "tensor", "achieved": round(achieved, 1), "peak": round(fp8_peak, 1), "unit": "TFLOP/s",
+                "frac": round(achieved / fp8_peak, 4), "traffic": None,
+                "kernel": "plane_gemm_tc_kernel<0> (residue GEMM, 3r FP8 plane products)",
+                "peak_source": f"{pk['source']} bf16 sustained x {FP8_TO_BF16} (nominal FP8/BF16 ratio)"}
+
+    # End to end through the public host-buffer entry: H2D of A and B, the
+    # emulated DGEMM, D2H of C, every step.
+    hA = torch.empty((w.k, w.m), dtype=torch.float64, pin_memory=True).t()   # column-major, pinned
+    hB = torch.empty((w.n, w.k), dtype=torch.float64, pin_memory=True).t()
+    hC = torch.empty((w.n, w.m), dtype=torch.float64, pin_memory=True).t()
+    hA.copy_(torch.from_numpy(A))
+    hB.copy_(torch.from_numpy(B))
+    e2e_steps = max(3, min(args.steps, 20))
+    oz.oz2_dgemm_host(hA, hB, hC, num_moduli=r)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        oz.oz2_dgemm_host(hA, hB, hC, num_moduli=r)
+    torch.cuda.synchronize()
+    e2e_s = (time.perf_counter() - t0) / e2e_steps
+    if world > 1:
+        t = torch.tensor([e2e_s], dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_s = float(t.item())
+    e2e = {"value": round(world * w.flops / e2e_s / 1e12, 3), "unit": "TFLOPS",
+           "h2d_bytes_per_step": in_bytes, "d2h_bytes_per_step": 8 * w.m * w.n,
+           "api": "oz2_dgemm_host (pinned host buffers)"}
+
+    extra = {}
+    if rank == 0:
+        # Accuracy on sampled rows: emulated (this r, and the r sweep) and native FP64.
+        rows = np.array([0, w.m // 2, w.m - 1])
+        C_host = dC.cpu().numpy()
+        extra["error"] = cref.scaled_error(C_host, A, B, rows=rows)
+        Cn = oz.oz2_native_dgemm(dA, dB)
+        extra["error_native_fp64"] = cref.scaled_error(Cn.cpu().numpy(), A, B, rows=rows)
+        if not args.no_sweep:
+            sweep = {}
+            for rr in range(6, 15):
+                Cr = oz.oz2_dgemm(dA, dB, num_moduli=rr)
+                sweep[str(rr)] = float(f"{cref.scaled_error(Cr.cpu().numpy(), A, B, rows=rows[:2]):.3e}")
+            extra["error_vs_r"] = sweep
+        if world == 1 and not args.no_cpu_baseline:
+            extra["cpu_baseline"] = cpu_baseline(w, r, A, B)
+
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+    if rank != 0:
+        return
+    out = {
+        "metric": METRIC, "value": round(value, 3), "unit": "TFLOPS", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "e4m3",
+        "data": "synthetic (seeded, a=U(-1/2,1/2)exp(phi N(0,1)))",
+        "config": {"workload": w.name, "m": w.m, "n": w.n, "k": w.k, "phi": w.phi, "num_moduli": r,
+                   "quant": "tz", "scale": "r2", "alpha": 3 * r + 1, "parallelism": f"replicas{world}",
+                   "l2": f"inputs {in_bytes / 2**20:.0f} MiB > L2 {L2_BYTES / 2**20:.0f} MiB"},
+        "clocks": sampler.summary(), "e2e": e2e, "gpu_launches": launches,
+        "roofline": roofline, "stages": stages,
+        "fp8_tensor_frac_of_alpha_roof": round(value * (3 * r + 1) / fp8_peak, 4),
+    }
+    out.update(extra)
+    print(json.dumps(out))
+
+
+def cpu_baseline(w, r, A, B, rows_per_sample=2):
+    """The oracle on the host cores: Phase 1 on the whole problem (scan, "+1"
+    pass, scales, quantisation, B's residues) plus Phases 2-3 for a few rows,
+    extrapolated linearly to all m rows."""
+    from oracle import ozaki2 as orc
+    t0 = time.perf_counter()
+    prep = orc.prepare(A, B, r)
+    t_phase1 = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    orc.evaluate_rows(prep, A, B, rows=np.arange(rows_per_sample))
+    t_rows = time.perf_counter() - t0
+    t_full = t_phase1 + t_rows * w.m / rows_per_sample
+    return {"value": round(w.flops / t_full / 1e12, 6), "unit": "TFLOPS", "cores": os.cpu_count(),
+            "kind": "oracle",
+            "sample": f"Phase 1 on the full {w.m}x{w.n}x{w.k} problem ({t_phase1:.1f} s) + Phases 2-3 on "
+                      f"{rows_per_sample} rows ({t_rows:.2f} s), extrapolated linearly to {w.m} rows; numpy "
+                      "BLAS threads for the exact integer matmuls, the rest single-threaded"}
+
+
+def run_reference(args):
+    """The oracle, timed on the host cores (rank 0 only)."""
+    world, rank, local = dist_env()
+    if rank != 0:
+        return
+    from oracle import ozaki2 as orc
+    w = wl.WORKLOADS[args.workload]
+    r = args.num_moduli
+    A, B = wl.make_inputs(w)
+    t0 = time.perf_counter()
+    prep = orc.prepare(A, B, r)
+    t_phase1 = time.perf_counter() - t0
+    rows_per_step = 1
+    # Each step: Phases 2-3 of one row plus that row's share of Phase 1.
+    share = t_phase1 * rows_per_step / w.m
+    for i in range(args.warmup):
+        orc.evaluate_rows(prep, A, B, rows=np.array([i % w.m]))
+    times = []
+    for i in range(args.steps):
+        t0 = time.perf_counter()
+        orc.evaluate_rows(prep, A, B, rows=np.array([(args.warmup + i) % w.m]))
+        times.append(time.perf_counter() - t0 + share)
+    step_s = max(sum(times) / len(times), 1e-9)
+    value = 2.0 * rows_per_step * w.n * w.k / step_s / 1e12
+    cb = {"value": round(value, 6), "unit": "TFLOPS", "cores": os.cpu_count(), "kind": "oracle",
+          "sample": f"each step: Phases 2-3 of one row of the {w.m}x{w.n}x{w.k} problem plus 1/{w.m} of the "
+                    f"measured full Phase 1 ({t_phase1:.1f} s)"}
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": round(value, 6), "unit": "TFLOPS", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(step_s * 1e3, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64",
+        "data": "synthetic (seeded)", "config": {"workload": w.name, "m": w.m, "n": w.n, "k": w.k, "phi": w.phi,
+                                                  "num_moduli": r},
+        "cpu_baseline": cb, "e2e": {"value": round(value, 6), "unit": "TFLOPS", "h2d_bytes_per_step": 0,
+                                    "d2h_bytes_per_step": 0}}))
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_oz2(args)
+
+
+if __name__ == "__main__":
+    main()

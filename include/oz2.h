@@ -1,0 +1,247 @@
+/*
+ * oz2.h -- C ABI of liboz2: FP64 matrix multiplication emulated with Ozaki
+ * Scheme II on FP8 (E4M3) tensor cores, for one NVIDIA GB300 (sm_103a).
+ *
+ * The method (arxiv 2606.06510, §2.3-2.5, Algorithm 1):
+ *   1. choose power-of-two row/column scales D, E and form the integer
+ *      matrices Ã = ⌊DA⌉, B̃ = ⌊BE⌉                          (Eq. scale)
+ *   2. for r pairwise-coprime moduli m_i, store the centred residues of Ã
+ *      and B̃ as E4M3 digit planes and form C^(i) = Ã B̃ mod m_i with three
+ *      FP8 plane products per modulus                 (Eq. modgemm, §2.5)
+ *   3. rebuild C̃ = ÃB̃ with Garner's algorithm and return D^-1 C̃ E^-1
+ *                                                      (Eq. garner, App. A)
+ * Rows of A (columns of B) holding a non-finite value, or whose exponent is
+ * far from the others, take a native FP64 path (Algorithm 1, fallback).
+ *
+ * Conventions shared by every entry point:
+ *  - Matrices are column-major, as in BLAS.  A is m×k (leading dimension
+ *    lda ≥ max(1,m)), B is k×n (ldb ≥ max(1,k)), C is m×n (ldc ≥ max(1,m)).
+ *  - Pointers named d_* are device pointers; h_* are host pointers.  The
+ *    caller owns every buffer it passes; the library never frees them.
+ *  - `stream` is a cudaStream_t (NULL = the legacy default stream).  Work is
+ *    enqueued asynchronously; no entry point synchronises the host on the
+ *    success path unless its comment says so.
+ *  - Return value: OZ2_OK or a negative oz2_status.  Errors detected on the
+ *    host are returned immediately and nothing is enqueued.  Errors raised by
+ *    a kernel (a bounded wait that timed out) are recorded in a device status
+ *    word read by oz2_get_stats()/oz2_check_device_status().
+ *  - num_moduli r ∈ [1, 16]: the first r moduli of the paper's set S
+ *    (1089, 1024, 961, 841, 625, 529, 511, 509, 503, 499, 491, 487; §2.5),
+ *    extended for r > 12 by 479, 467, 463, 461.  r = 12 is the paper's
+ *    working point; r = 13 is needed for FP64-level accuracy at large k.
+ */
+#ifndef OZ2_H
+#define OZ2_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  OZ2_OK = 0,
+  OZ2_ERR_INVALID_ARG = -1,   /* a size, leading dimension or pointer is invalid */
+  OZ2_ERR_UNSUPPORTED_R = -2, /* num_moduli outside [1, 16] */
+  OZ2_ERR_ALLOC = -3,         /* workspace allocation failed or too small */
+  OZ2_ERR_CUDA = -4,          /* a CUDA runtime call or launch failed */
+  OZ2_ERR_TIMEOUT = -5,       /* a device-side bounded wait expired */
+  OZ2_ERR_UNSUPPORTED = -6    /* a size beyond the implemented limits */
+} oz2_status;
+
+/* Quantiser of Eq. (scale), Table "numerical-contract variants". */
+typedef enum { OZ2_QUANT_TZ = 0, OZ2_QUANT_RN = 1 } oz2_quant;
+
+/* Scale choice.  R2 (default): per-row/column power-of-two scales from the
+ * "+1" max-magnitude GEMM U = ÂB̂ (§2.4), so that Σ_l|Ã_il||B̃_lj| ≤ 2^T < M/2.
+ * R1: the crude bound μ = k·max|Ã|·max|B̃| of Algorithm 1 (no "+1" GEMM). */
+typedef enum { OZ2_SCALE_R2 = 0, OZ2_SCALE_R1 = 1 } oz2_scale_mode;
+
+/* Flags for oz2_dgemm_ex. */
+#define OZ2_FLAG_NO_FALLBACK 0x1u   /* flag only non-finite rows/columns */
+#define OZ2_FLAG_TIMING      0x2u   /* record per-stage CUDA events on the stream;
+                                       harvested by oz2_get_stats (no host sync
+                                       inside the call) */
+/* Diagnostic only: run the "+1" and residue plane GEMMs on CUDA cores with
+ * the same integer plane products and epilogue arithmetic (slow; used by
+ * the tests to separate tensor-core issues from the rest of the path). */
+#define OZ2_FLAG_DEBUG_SIMT_GEMM 0x100u
+
+/* Statistics of the most recent oz2_dgemm / oz2_dgemm_ex call on this
+ * device.  Reading them synchronises the device. */
+typedef struct {
+  int32_t status;            /* device status word: 0, or an oz2_status */
+  int32_t fallback_rows;     /* rows of A that took the native FP64 path */
+  int32_t fallback_cols;     /* columns of B that took the native FP64 path */
+  int32_t u_max;             /* max_i u_i of the "+1" pass (R2) */
+  int32_t s;                 /* common column budget s (R2), or pB (R1) */
+  int32_t d_min, d_max;      /* range of the row exponents d_i */
+  int32_t e_min, e_max;      /* range of the column exponents e_j */
+  int32_t k_slab;            /* K-slab of exact FP32 accumulation used */
+  float stage_ms[8];         /* mean per call of: scan, magnitude planes,
+                                "+1" GEMM, scale choice, deconstruct, residue
+                                GEMM, CRT, fallback -- over the calls made
+                                with OZ2_FLAG_TIMING since the last read */
+  int32_t timed_calls;       /* number of calls averaged in stage_ms */
+  int64_t kernel_launches;   /* kernels launched by the library since the
+                                last read (all devices) */
+} oz2_stats;
+
+/* ---------------------------------------------------------------------
+ * Production entry points
+ * ------------------------------------------------------------------- */
+
+/* C = A·B (overwrite, β = 0) by Ozaki Scheme II with TZ quantiser and R2
+ * scales.  Allocates its workspace with cudaMallocAsync on `stream` and
+ * frees it on the same stream.  m == 0 or n == 0: no-op; k == 0: C = 0. */
+int oz2_dgemm(int64_t m, int64_t n, int64_t k,
+              const double* d_A, int64_t lda,
+              const double* d_B, int64_t ldb,
+              double* d_C, int64_t ldc,
+              int num_moduli, void* stream);
+
+/* As oz2_dgemm with A, B and C in HOST memory (pinned memory gives the
+ * best transfer rate).  Copies A and B to the device, computes, copies C
+ * back, and synchronises `stream` before returning.  Device buffers and the
+ * workspace are allocated and freed stream-ordered inside the call. */
+int oz2_dgemm_host(int64_t m, int64_t n, int64_t k,
+                   const double* h_A, int64_t lda,
+                   const double* h_B, int64_t ldb,
+                   double* h_C, int64_t ldc,
+                   int num_moduli, void* stream);
+
+/* Bytes of device workspace oz2_dgemm_ex needs for this problem. */
+size_t oz2_workspace_size(int64_t m, int64_t n, int64_t k, int num_moduli);
+
+/* As oz2_dgemm, with an explicit quantiser (oz2_quant), scale mode
+ * (oz2_scale_mode), flags (OZ2_FLAG_*) and caller-provided device workspace of
+ * ws_bytes ≥ oz2_workspace_size(...) bytes, 256-byte aligned.  After the
+ * call the workspace holds the intermediates at the offsets reported by
+ * oz2_workspace_layout (they stay valid until the workspace is reused). */
+int oz2_dgemm_ex(int64_t m, int64_t n, int64_t k,
+                 const double* d_A, int64_t lda,
+                 const double* d_B, int64_t ldb,
+                 double* d_C, int64_t ldc,
+                 int num_moduli, int quant, int scale, unsigned flags,
+                 void* d_workspace, size_t ws_bytes, void* stream);
+
+/* Byte offsets of the intermediates inside the oz2_dgemm_ex workspace.
+ * Layouts (all written by the library):
+ *   ra[m], cb[n]          int32  row/column max-exponents (|x| < 2^e)
+ *   row_flag[m], col_flag[n] uint8  bit0 fallback, bit1 zero in emulation
+ *   d[m], e[n]            int32  the scale exponents (D = diag 2^d_i ...)
+ *   urow[m]               float  max_j U_ij of the "+1" GEMM (R2)
+ *   mag_a, mag_b          uint8  magnitude planes Â (m×k_pad), B̂ (n×k_pad)
+ *   planes_a, planes_b    uint8  E4M3 digit planes, see oz2_plane_layout
+ *   residues              int16  r matrices C^(i), each m×n column-major
+ *                                (ld = m), centred in [-⌊m_i/2⌋, m_i-1-⌊m_i/2⌋]
+ */
+typedef struct {
+  size_t ra, cb, row_flag, col_flag, d, e, urow, misc;
+  size_t mag_a, mag_b, planes_a, planes_b, residues, total;
+  int64_t k_pad;             /* k rounded up to a multiple of 128 */
+  int32_t num_planes;        /* stored planes per operand element */
+} oz2_ws_layout;
+int oz2_workspace_layout(int64_t m, int64_t n, int64_t k, int num_moduli,
+                         oz2_ws_layout* out);
+
+/* Digit-plane layout (§2.5).  For operand X with `rows` rows (m for A, n
+ * for B) every plane is a rows×k_pad byte matrix, row-major (k contiguous),
+ * zero-padded from k to k_pad; plane p starts at byte p·rows·k_pad.  The
+ * planes of modulus i are consecutive, starting at plane_offset[i]:
+ *   square m_i = s²:  (d0, d1)            d = d0 + s·d1, balanced base s
+ *   nonsquare:        (d0+d1, d0, d1)     d = d0 + 16·d1, carry-corrected
+ * where d is the centred residue of the integer Ã (or B̃) entry.  Each byte
+ * is the E4M3 code of the integer digit.  Writes num_moduli offsets and
+ * returns the total plane count. */
+int oz2_plane_layout(int num_moduli, int32_t* plane_offset);
+
+/* Statistics of the last call on the current device (synchronises; resets
+ * the timing accumulators and the launch counter). */
+int oz2_get_stats(oz2_stats* out);
+
+/* Synchronises the device and returns the device status word (OZ2_OK or
+ * OZ2_ERR_TIMEOUT), clearing it. */
+int oz2_check_device_status(void);
+
+/* Human-readable name of an oz2_status. */
+const char* oz2_status_string(int status);
+
+/* ---------------------------------------------------------------------
+ * Stage entry points (the same kernels the production path runs).  They
+ * exist so that each stage can be checked against the CPU oracle alone.
+ * ------------------------------------------------------------------- */
+
+/* Stage 1a (Algorithm 1 "scan the exponent spans"): row max-exponents of A
+ * and column max-exponents of B, non-finite detection, and the fallback
+ * flags (non-finite, or max-exponent more than 128 binades from the lower
+ * median of the nonzero rows).  Outputs as in oz2_ws_layout. */
+int oz2_scan(int64_t m, int64_t n, int64_t k,
+             const double* d_A, int64_t lda, const double* d_B, int64_t ldb,
+             unsigned flags, int32_t* d_ra, int32_t* d_cb,
+             uint8_t* d_row_flag, uint8_t* d_col_flag, void* stream);
+
+/* Stage 1b+2' (§2.4, "+1" pass): magnitude planes Â_il = 2^max(-c, ⌈log2
+ * |A_il|2^-ra_i⌉) (E4M3, m×k_pad and n×k_pad as the digit planes), the
+ * FP8 GEMM U = ÂB̂ (exact in FP32), and the exponents d[m], e[n]
+ * (oz2_scale_mode).  d_urow receives max_j U_ij.  d_mag_a/d_mag_b are outputs. */
+int oz2_scale(int64_t m, int64_t n, int64_t k, int num_moduli,
+              const double* d_A, int64_t lda, const double* d_B, int64_t ldb,
+              const int32_t* d_ra, const int32_t* d_cb,
+              const uint8_t* d_row_flag, const uint8_t* d_col_flag,
+              int quant, int scale, uint8_t* d_mag_a, uint8_t* d_mag_b,
+              float* d_urow, int32_t* d_d, int32_t* d_e, void* stream);
+
+/* Stage 3 (Eq. scale and Algorithm 1 "lin:dec"): Ã = ⌊2^d_i A_il⌉ and
+ * B̃ = ⌊2^e_j B_lj⌉, their centred residues, and the E4M3 digit planes in
+ * the oz2_plane_layout order.  Rows with row_flag bit1 (columns with
+ * col_flag bit1) are written as zero. */
+int oz2_deconstruct(int64_t m, int64_t n, int64_t k, int num_moduli,
+                    const double* d_A, int64_t lda, const double* d_B, int64_t ldb,
+                    const int32_t* d_d, const int32_t* d_e,
+                    const uint8_t* d_row_flag, const uint8_t* d_col_flag,
+                    int quant, uint8_t* d_planes_a, uint8_t* d_planes_b,
+                    void* stream);
+
+/* Stage 4 (Eq. modgemm, Eq. sq-shortcut, Eq. kar): from digit planes in
+ * the oz2_plane_layout order (k_pad = k rounded up to 128), the residue
+ * matrices C^(i) = (A^(i) B^(i)) mod m_i, centred, r × (m×n column-major,
+ * ld = m) int16.  Three FP8 tcgen05 MMAs per modulus with exact FP32
+ * accumulation (Eq. accum-exact), reduced mod m_i every K-slab. */
+int oz2_residue_gemm(int64_t m, int64_t n, int64_t k, int num_moduli,
+                     const uint8_t* d_planes_a, const uint8_t* d_planes_b,
+                     int16_t* d_residues, void* stream);
+
+/* Diagnostic twin of oz2_residue_gemm on CUDA cores (same products, same
+ * epilogue arithmetic, sequential k order); slow. */
+int oz2_residue_gemm_simt(int64_t m, int64_t n, int64_t k, int num_moduli,
+                          const uint8_t* d_planes_a, const uint8_t* d_planes_b,
+                          int16_t* d_residues, void* stream);
+
+/* Stage 5 (Eq. garner, App. A; Algorithm 1 unscale): C_ij = RN_fp64(X_ij ·
+ * 2^-(d_i+e_j)) with X_ij ∈ [-M/2, M/2) the integer whose residues are
+ * C^(i)_ij.  residues: r × (m×n, ld = ldr) int16, centred or not. */
+int oz2_reconstruct(int64_t m, int64_t n, int num_moduli,
+                    const int16_t* d_residues, int64_t ldr,
+                    const int32_t* d_d, const int32_t* d_e,
+                    double* d_C, int64_t ldc, void* stream);
+
+/* Stage 6 (Algorithm 1, native fallback): for every row i with row_flag
+ * bit0 and every column j with col_flag bit0, C_ij = the FP64 FMA chain
+ * Σ_l A_il B_lj in the order l = 0..k-1, starting from +0. */
+int oz2_fallback(int64_t m, int64_t n, int64_t k,
+                 const double* d_A, int64_t lda, const double* d_B, int64_t ldb,
+                 const uint8_t* d_row_flag, const uint8_t* d_col_flag,
+                 double* d_C, int64_t ldc, void* stream);
+
+/* The native-FP64 comparator: C = A·B with every entry the FMA chain of
+ * oz2_fallback (no emulation). */
+int oz2_native_dgemm(int64_t m, int64_t n, int64_t k,
+                     const double* d_A, int64_t lda, const double* d_B, int64_t ldb,
+                     double* d_C, int64_t ldc, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* OZ2_H */

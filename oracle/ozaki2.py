@@ -542,9 +542,13 @@ class Result:
     extra: dict = field(default_factory=dict)
 
 
-def oz2_dgemm(A, B, r: int = 12, quant: str = "tz", scale: str = "r2",
-              fallback: bool = True) -> Result:
-    """C ≈ AB by Ozaki Scheme II (Algorithm 1), every intermediate returned."""
+def prepare(A, B, r: int = 12, quant: str = "tz", scale: str = "r2", fallback: bool = True) -> Result:
+    """Phase 1 of Algorithm 1 and the scale choice, on the whole problem.
+
+    Returns a Result without C: exponents, flags, the "+1" pass, d, e, the
+    integer matrices Ã, B̃ (Eq. scale) and the centred residues of B̃ for each
+    modulus (Algorithm 1 "lin:dec" for B, needed by every row of C).
+    """
     A = np.asarray(A, dtype=np.float64)
     B = np.asarray(B, dtype=np.float64)
     m, k = A.shape
@@ -584,26 +588,60 @@ def oz2_dgemm(A, B, r: int = 12, quant: str = "tz", scale: str = "r2",
     res.d, res.e = d, e
 
     # Eq. (scale): integer matrices (flagged rows/columns are zero here).
-    At = quantise(np.where(zero_rows[:, None], 0.0, A), d, quant)
-    Bt = quantise(np.where(zero_cols[:, None], 0.0, B.T), e, quant).T
-    res.At, res.Bt = At, Bt
-
-    # Phase 2: modular GEMMs.  Phase 3: Garner and unscale.
-    R = residue_products(At, Bt, mods)
-    X = garner_value(R, mods)
-    C = unscale(X, d, e)
-    res.residues, res.X = R, X
-
-    # Native FP64 on flagged rows and columns.
-    for i in np.flatnonzero(row_flag):
-        for j in range(n):
-            C[i, j] = native_entry(A, B, i, j)
-    for j in np.flatnonzero(col_flag):
-        for i in range(m):
-            if not row_flag[i]:
-                C[i, j] = native_entry(A, B, i, j)
-    res.C = C
+    res.At = quantise(np.where(zero_rows[:, None], 0.0, A), d, quant)
+    res.Bt = quantise(np.where(zero_cols[:, None], 0.0, B.T), e, quant).T
+    # Centred residues of B̃, held as float64 (exact: |residue| ≤ 544) with
+    # the bound of exact_int_matmul checked once here.
+    bres = []
+    for mi in mods:
+        b = centred(res.Bt, mi)
+        h = mi - mi // 2
+        assert np.abs(b).max(initial=0) <= h and k * h * h < 2**53
+        bres.append(b.astype(np.float64))
+    res.extra["b_residues"] = bres
     return res
+
+
+def evaluate_rows(prep: Result, A, B, rows=None) -> Result:
+    """Phases 2-3 (Eq. modgemm, Eq. garner, unscale) and the native fallback
+    for the given rows of C (all rows when ``rows`` is None)."""
+    A = np.asarray(A, dtype=np.float64)
+    B = np.asarray(B, dtype=np.float64)
+    m, n = A.shape[0], B.shape[1]
+    mods = prep.mods
+    sel = np.arange(m) if rows is None else np.asarray(rows, dtype=np.int64)
+    At = prep.At[sel]
+    out = []
+    for mi, b in zip(mods, prep.extra["b_residues"]):
+        # exact: every partial sum is an integer below k·(m/2)^2 < 2^53
+        a = centred(At, mi).astype(np.float64)
+        out.append(centred((a @ b).astype(np.int64), mi))
+    R = np.stack(out) if out else np.zeros((0, sel.size, n), np.int64)
+    X = garner_value(R, mods)
+    C = unscale(X, prep.d[sel], prep.e)
+    # Native FP64 on flagged rows and columns.
+    for a, i in enumerate(sel):
+        if prep.row_flag[i]:
+            for j in range(n):
+                C[a, j] = native_entry(A, B, i, j)
+    for j in np.flatnonzero(prep.col_flag):
+        for a, i in enumerate(sel):
+            if not prep.row_flag[i]:
+                C[a, j] = native_entry(A, B, i, j)
+    res = Result(**{f: getattr(prep, f) for f in prep.__dataclass_fields__})
+    res.residues, res.X, res.C = R, X, C
+    return res
+
+
+def oz2_dgemm(A, B, r: int = 12, quant: str = "tz", scale: str = "r2",
+              fallback: bool = True, rows=None) -> Result:
+    """C ≈ AB by Ozaki Scheme II (Algorithm 1), every intermediate returned.
+
+    With ``rows`` (an index array) Phase 1 and the scale choice still run on
+    the whole problem, but Phases 2-3 and the fallback are evaluated only for
+    those rows of C (``C``, ``residues`` and ``X`` then hold those rows).
+    """
+    return evaluate_rows(prepare(A, B, r, quant, scale, fallback), A, B, rows)
 
 
 def truncation_bound(A, B, d, e, quant: str = "tz"):

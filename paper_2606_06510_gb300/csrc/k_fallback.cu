@@ -1,0 +1,130 @@
+// Native-FP64 fallback (Algorithm 1, the "if" on admissibility; §2.6 contract
+// item (vi)): rows of A (columns of B) flagged by the scan are recomputed
+// with FP64 FMA chains, every output C_ij = fma(A_i,k-1, B_k-1,j, ... fma(A_i0,
+// B_0j, +0)), in the order l = 0..k-1, so the result is reproducible.
+//
+// Tiled CUDA-core DGEMM over index lists: 64×64 output tiles, 256 threads,
+// 4×4 outputs per thread, k staged through shared memory in chunks of 16.
+// The same kernel is the cuBLAS-free native comparator (identity lists).
+#include "oz2_common.cuh"
+
+namespace oz2 {
+
+constexpr int kFT = 64, kFK = 16;
+
+// Compact the indices whose flag has bit0 set into `list`, counting in *count.
+__global__ void compact_flags_kernel(int64_t cnt, const uint8_t* __restrict__ flag, int* __restrict__ list,
+                                     int* __restrict__ count) {
+  int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (i < cnt && (flag[i] & 1)) list[atomicAdd(count, 1)] = static_cast<int>(i);
+}
+
+// rows: row_list ? row_list[0..*row_count) : 0..m-1 ; cols likewise.
+__global__ void __launch_bounds__(256) fma_gemm_kernel(int64_t m, int64_t n, int64_t k,
+                                                       const double* __restrict__ A, int64_t lda,
+                                                       const double* __restrict__ B, int64_t ldb,
+                                                       const int* __restrict__ row_list,
+                                                       const int* __restrict__ row_count,
+                                                       const int* __restrict__ col_list,
+                                                       const int* __restrict__ col_count, double* __restrict__ C,
+                                                       int64_t ldc) {
+  __shared__ double As[kFK][kFT + 1];
+  __shared__ double Bs[kFK][kFT + 1];
+  __shared__ int rid[kFT], cid[kFT];
+  const int64_t nr = row_list ? *row_count : m;
+  const int64_t nc = col_list ? *col_count : n;
+  const int64_t rt = (nr + kFT - 1) / kFT, ct = (nc + kFT - 1) / kFT;
+  const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+  for (int64_t tile = blockIdx.x; tile < rt * ct; tile += gridDim.x) {
+    const int64_t r0 = (tile % rt) * kFT, c0 = (tile / rt) * kFT;
+    __syncthreads();
+    if (threadIdx.x < kFT) {
+      const int64_t a = r0 + threadIdx.x;
+      rid[threadIdx.x] = a < nr ? (row_list ? row_list[a] : static_cast<int>(a)) : -1;
+    } else if (threadIdx.x < 2 * kFT) {
+      const int64_t b = c0 + threadIdx.x - kFT;
+      cid[threadIdx.x - kFT] = b < nc ? (col_list ? col_list[b] : static_cast<int>(b)) : -1;
+    }
+    __syncthreads();
+    double acc[4][4];
+#pragma unroll
+    for (int a = 0; a < 4; ++a)
+#pragma unroll
+      for (int b = 0; b < 4; ++b) acc[a][b] = 0.0;
+    for (int64_t l0 = 0; l0 < k; l0 += kFK) {
+      __syncthreads();
+      // A tile: 64 rows × 16 k; thread loads 4 entries (row = t % 64, k = t / 64 + 4q).
+      for (int q = 0; q < 4; ++q) {
+        const int rr = threadIdx.x & 63, kk = (threadIdx.x >> 6) + 4 * q;
+        const int gi = rid[rr];
+        const int64_t l = l0 + kk;
+        As[kk][rr] = (gi >= 0 && l < k) ? A[gi + l * lda] : 0.0;
+        const int cc = threadIdx.x & 63;
+        const int gj = cid[cc];
+        // B tile: 16 k × 64 cols; same pattern (k fastest would coalesce better;
+        // the fallback is rare and small).
+        Bs[kk][cc] = (gj >= 0 && l < k) ? B[l + gj * ldb] : 0.0;
+      }
+      __syncthreads();
+      const int kmax = static_cast<int>(k - l0 < kFK ? k - l0 : kFK);
+      for (int kk = 0; kk < kmax; ++kk) {
+        double av[4], bv[4];
+#pragma unroll
+        for (int a = 0; a < 4; ++a) av[a] = As[kk][ty * 4 + a];
+#pragma unroll
+        for (int b = 0; b < 4; ++b) bv[b] = Bs[kk][tx * 4 + b];
+#pragma unroll
+        for (int a = 0; a < 4; ++a)
+#pragma unroll
+          for (int b = 0; b < 4; ++b) acc[a][b] = fma(av[a], bv[b], acc[a][b]);
+      }
+    }
+#pragma unroll
+    for (int a = 0; a < 4; ++a) {
+      const int gi = rid[ty * 4 + a];
+      if (gi < 0) continue;
+#pragma unroll
+      for (int b = 0; b < 4; ++b) {
+        const int gj = cid[tx * 4 + b];
+        if (gj >= 0) C[gi + static_cast<int64_t>(gj) * ldc] = acc[a][b];
+      }
+    }
+  }
+}
+
+static int fb_grid() {
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  return sms * 4;
+}
+
+// scratch: (m + n + 2) ints of device memory (lists and counts).
+cudaError_t launch_fallback_lists(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, const double* B,
+                                  int64_t ldb, const uint8_t* row_flag, const uint8_t* col_flag, int* scratch,
+                                  double* C, int64_t ldc, cudaStream_t st) {
+  if (m == 0 || n == 0) return cudaSuccess;
+  int* counts = scratch;              // [0]: rows, [1]: cols
+  int* rlist = scratch + 2;
+  int* clist = rlist + m;
+  cudaError_t err = cudaMemsetAsync(counts, 0, 2 * sizeof(int), st);
+  if (err != cudaSuccess) return err;
+  count_launch(4);
+  compact_flags_kernel<<<static_cast<unsigned>((m + 255) / 256), 256, 0, st>>>(m, row_flag, rlist, counts);
+  compact_flags_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, st>>>(n, col_flag, clist, counts + 1);
+  const int g = fb_grid();
+  // flagged rows × all columns, then all rows × flagged columns
+  fma_gemm_kernel<<<g, 256, 0, st>>>(m, n, k, A, lda, B, ldb, rlist, counts, nullptr, nullptr, C, ldc);
+  fma_gemm_kernel<<<g, 256, 0, st>>>(m, n, k, A, lda, B, ldb, nullptr, nullptr, clist, counts + 1, C, ldc);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_native(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, const double* B,
+                          int64_t ldb, double* C, int64_t ldc, cudaStream_t st) {
+  if (m == 0 || n == 0) return cudaSuccess;
+  count_launch();
+  fma_gemm_kernel<<<fb_grid(), 256, 0, st>>>(m, n, k, A, lda, B, ldb, nullptr, nullptr, nullptr, nullptr, C, ldc);
+  return cudaGetLastError();
+}
+
+}  // namespace oz2

@@ -1,0 +1,658 @@
+// C ABI of liboz2 (declared in include/oz2.h): argument checks, the modulus
+// constants and digit-plane table, workspace carving, and the stage order of
+// Algorithm 1 (scan → "+1" pass and scales → deconstruct → residue GEMMs →
+// Garner/unscale → native fallback).
+#include <algorithm>
+#include <atomic>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+
+#include "oz2_common.cuh"
+
+namespace oz2 {
+
+// §2.5: the published set S (six squares, then the nonsquare tail), then the
+// extension primes used for r = 13..16 (nonsquare, < 513).
+static const int kModuliAll[kMaxModuli] = {1089, 1024, 961, 841, 625, 529, 511, 509,
+                                           503,  499,  491, 487, 479, 467, 463, 461};
+constexpr int kTableMax = 10240;  // Σ of all sixteen moduli = 9939 entries
+
+// Packed E4M3 digit planes of every residue (byte p = plane p), per modulus.
+static __device__ uint32_t g_plane_table[kTableMax];
+// Device status block (sticky status word, fallback counts, scale summary).
+static __device__ Oz2Device g_status;
+
+// ---------------------------------------------------------------------------
+// Host-side arithmetic for the constants.
+// ---------------------------------------------------------------------------
+static int isqrt_exact(int m) {
+  for (int s = 1; s * s <= m; ++s)
+    if (s * s == m) return s;
+  return 0;
+}
+
+// E4M3-exact integers: M·2^e with |M| ≤ 15 and magnitude ≤ 448 (§2.5).
+static bool e4m3_exact(int v) {
+  int a = v < 0 ? -v : v;
+  if (a == 0) return true;
+  if (a > 448) return false;
+  while ((a & 1) == 0) a >>= 1;
+  return a <= 15;
+}
+
+// E4M3 byte: sign | (e+7) << 3 | fraction, for an integer in 𝔼.
+static uint8_t e4m3_code(int v) {
+  if (v == 0) return 0;
+  int a = v < 0 ? -v : v;
+  int e = 31 - __builtin_clz(static_cast<unsigned>(a));
+  int frac = ((a << 3) >> e) - 8;
+  return static_cast<uint8_t>((v < 0 ? 0x80 : 0) | ((e + 7) << 3) | frac);
+}
+
+static int floor_mod(int a, int m) {
+  int r = a % m;
+  return r < 0 ? r + m : r;
+}
+
+// Digit planes of the centred residue d (§2.5).
+static uint32_t plane_word(int d, int m) {
+  int s = isqrt_exact(m);
+  int p[3] = {0, 0, 0}, np;
+  if (s) {  // balanced base s: d0 ∈ [-⌊s/2⌋, s-1-⌊s/2⌋]
+    int h = s / 2;
+    int d0 = floor_mod(d + h, s) - h;
+    int d1 = (d - d0) / s;
+    p[0] = d0;
+    p[1] = d1;
+    np = 2;
+  } else {  // balanced base 16 with the carry correction
+    int d0 = floor_mod(d + 8, 16) - 8;
+    int d1 = (d - d0) / 16;
+    if (!e4m3_exact(d0 + d1)) {
+      int sg = d0 > 0 ? 1 : -1;
+      d0 -= 16 * sg;
+      d1 += sg;
+    }
+    p[0] = d0 + d1;
+    p[1] = d0;
+    p[2] = d1;
+    np = 3;
+  }
+  uint32_t w = 0;
+  for (int i = 0; i < np; ++i) {
+    if (!e4m3_exact(p[i])) {
+      std::fprintf(stderr, "oz2: digit %d of residue %d mod %d is not E4M3-exact\n", p[i], d, m);
+      return 0xFFFFFFFFu;
+    }
+    w |= static_cast<uint32_t>(e4m3_code(p[i])) << (8 * i);
+  }
+  return w;
+}
+
+static int mod_inverse(long long a, int m) {
+  long long t = 0, nt = 1, r = m, nr = floor_mod(static_cast<int>(a % m), m);
+  while (nr) {
+    long long q = r / nr, tmp;
+    tmp = t - q * nt; t = nt; nt = tmp;
+    tmp = r - q * nr; r = nr; nr = tmp;
+  }
+  return static_cast<int>(t < 0 ? t + m : t);
+}
+
+typedef unsigned long long u64;
+static void mul3(u64 (&x)[3], u64 m) {
+  unsigned __int128 c = 0;
+  for (int i = 0; i < 3; ++i) {
+    unsigned __int128 p = static_cast<unsigned __int128>(x[i]) * m + c;
+    x[i] = static_cast<u64>(p);
+    c = p >> 64;
+  }
+}
+static int bitlen3(const u64 (&x)[3]) {
+  for (int i = 2; i >= 0; --i)
+    if (x[i]) return 64 * i + 64 - __builtin_clzll(x[i]);
+  return 0;
+}
+
+static Oz2Moduli build_moduli(int r, int quant) {
+  Oz2Moduli c;
+  std::memset(&c, 0, sizeof(c));
+  c.r = r;
+  int plane = 0, toff = 0;
+  for (int i = 0; i < r; ++i) {
+    const int m = kModuliAll[i];
+    c.m[i] = m;
+    c.sq_base[i] = isqrt_exact(m);
+    c.plane_off[i] = plane;
+    plane += c.sq_base[i] ? 2 : 3;
+    c.table_off[i] = toff;
+    toff += m;
+    int sh = 31 - __builtin_clz(static_cast<unsigned>(m - 1));
+    u64 num = 1ull << (32 + sh);
+    c.magic[i] = static_cast<uint32_t>((num + m - 1) / m);
+    c.magic_sh[i] = sh;
+    for (int j = 0; j < 4; ++j) {
+      u64 v = 1;
+      for (int t = 0; t < j; ++t) v = (v << 16) % m;
+      c.limb[i][j] = static_cast<int>(v);
+    }
+    c.negoff[i] = m * static_cast<int>(((1u << 28) + m - 1) / m);
+    c.goff[i] = m * static_cast<int>(((1u << 27) + m - 1) / m);
+    long long P = 1;  // product of the earlier moduli, mod m
+    for (int t = 0; t < i; ++t) {
+      c.pmod[i][t] = static_cast<int>(P);
+      P = (P * kModuliAll[t]) % m;
+    }
+    c.inv[i] = i ? mod_inverse(P, m) : 1;
+  }
+  c.nplanes = plane;
+  c.table_entries = toff;
+  u64 M[3] = {1, 0, 0};
+  for (int i = 0; i < r; ++i) mul3(M, static_cast<u64>(kModuliAll[i]));
+  for (int i = 0; i < 3; ++i) c.M[i] = M[i];
+  // ⌈M/2⌉ = (M + 1) >> 1
+  u64 Mp[3] = {M[0] + 1, M[1] + (M[0] + 1 == 0), M[2]};
+  c.Mhalf[0] = (Mp[0] >> 1) | (Mp[1] << 63);
+  c.Mhalf[1] = (Mp[1] >> 1) | (Mp[2] << 63);
+  c.Mhalf[2] = Mp[2] >> 1;
+  // TZ: largest T with 2^(T+1) < M, i.e. bitlen(M-1) - 2; RN two bits less.
+  u64 Mm1[3] = {M[0] - 1, M[1] - (M[0] == 0), M[2]};
+  int t_tz = bitlen3(Mm1) - 2;
+  c.T = quant == OZ2_QUANT_RN ? t_tz - 2 : t_tz;
+  return c;
+}
+
+// ---------------------------------------------------------------------------
+// Per-device state: the plane table is uploaded once per device.
+// ---------------------------------------------------------------------------
+struct DeviceState {
+  bool ready = false;
+  uint32_t* table = nullptr;
+  Oz2Device* status = nullptr;
+};
+static DeviceState g_devs[64];
+static std::mutex g_mu;
+
+// Per-stage timing: each timed call records 9 events into one set of a
+// ring; sets are harvested (synchronised) when stats are read or when the
+// ring wraps onto a set still pending.
+constexpr int kTimingSets = 32;
+struct TimingSet {
+  cudaEvent_t ev[9];
+  bool created = false;
+  bool pending = false;
+};
+struct HostStats {
+  int k_slab = 0;
+  double stage_sum[8] = {0};
+  int timed = 0;
+  TimingSet sets[kTimingSets];
+  int next = 0;
+};
+static HostStats g_host_stats[64];
+static std::atomic<long long> g_launches{0};
+
+static void harvest(HostStats& hs, TimingSet& t) {
+  if (!t.pending) return;
+  if (cudaEventSynchronize(t.ev[8]) == cudaSuccess) {
+    for (int i = 0; i < 8; ++i) {
+      float ms = 0.f;
+      cudaEventElapsedTime(&ms, t.ev[i], t.ev[i + 1]);
+      hs.stage_sum[i] += ms;
+    }
+    ++hs.timed;
+  }
+  t.pending = false;
+}
+
+static int device_state(DeviceState** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return OZ2_ERR_CUDA;
+  std::lock_guard<std::mutex> lk(g_mu);
+  DeviceState& s = g_devs[dev];
+  if (!s.ready) {
+    static uint32_t host_table[kTableMax];
+    int off = 0;
+    for (int i = 0; i < kMaxModuli; ++i) {
+      const int m = kModuliAll[i];
+      for (int r = 0; r < m; ++r) {
+        int d = r > m - 1 - m / 2 ? r - m : r;  // centred residue
+        uint32_t w = plane_word(d, m);
+        if (w == 0xFFFFFFFFu) return OZ2_ERR_CUDA;
+        host_table[off + r] = w;
+      }
+      off += m;
+    }
+    if (cudaMemcpyToSymbol(g_plane_table, host_table, sizeof(uint32_t) * off) != cudaSuccess)
+      return OZ2_ERR_CUDA;
+    Oz2Device zero;
+    std::memset(&zero, 0, sizeof(zero));
+    if (cudaMemcpyToSymbol(g_status, &zero, sizeof(zero)) != cudaSuccess) return OZ2_ERR_CUDA;
+    if (cudaGetSymbolAddress(reinterpret_cast<void**>(&s.table), g_plane_table) != cudaSuccess ||
+        cudaGetSymbolAddress(reinterpret_cast<void**>(&s.status), g_status) != cudaSuccess)
+      return OZ2_ERR_CUDA;
+    s.ready = true;
+  }
+  *out = &s;
+  return OZ2_OK;
+}
+
+__global__ void reset_status_kernel(Oz2Device* dev) {
+  dev->fallback_rows = 0;
+  dev->fallback_cols = 0;
+  dev->u_max_bits = 0;
+  dev->s = 0;
+}
+
+void count_launch(int n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+
+static size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+static void compute_layout(int64_t m, int64_t n, int64_t k, int r, oz2_ws_layout* L) {
+  const int64_t k_pad = (k + kKPad - 1) / kKPad * kKPad;
+  int planes = 0;
+  for (int i = 0; i < r; ++i) planes += isqrt_exact(kModuliAll[i]) ? 2 : 3;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    size_t o = off;
+    off = align256(off + bytes);
+    return o;
+  };
+  L->ra = take(4 * m);
+  L->cb = take(4 * n);
+  L->row_flag = take(m);
+  L->col_flag = take(n);
+  L->d = take(4 * m);
+  L->e = take(4 * n);
+  L->urow = take(4 * m);
+  L->misc = take(4 * (m + n + 2));
+  L->mag_a = take(static_cast<size_t>(m) * k_pad);
+  L->mag_b = take(static_cast<size_t>(n) * k_pad);
+  L->planes_a = take(static_cast<size_t>(planes) * m * k_pad);
+  L->planes_b = take(static_cast<size_t>(planes) * n * k_pad);
+  L->residues = take(2 * static_cast<size_t>(r) * m * n);
+  L->total = off;
+  L->k_pad = k_pad;
+  L->num_planes = planes;
+}
+
+static int check_sizes(int64_t m, int64_t n, int64_t k, int64_t lda, int64_t ldb, int64_t ldc) {
+  if (m < 0 || n < 0 || k < 0) return OZ2_ERR_INVALID_ARG;
+  if (lda < std::max<int64_t>(1, m) || ldb < std::max<int64_t>(1, k) || ldc < std::max<int64_t>(1, m))
+    return OZ2_ERR_INVALID_ARG;
+  // Tile coordinates are 32-bit; U·2^2c ≤ k·2^2c ≤ 2^24 needs k ≤ 2^24.
+  if (m >= (1LL << 31) || n >= (1LL << 31) || k > (1LL << 24)) return OZ2_ERR_UNSUPPORTED;
+  return OZ2_OK;
+}
+
+static int to_status(cudaError_t e) { return e == cudaSuccess ? OZ2_OK : OZ2_ERR_CUDA; }
+
+}  // namespace oz2
+
+using namespace oz2;
+
+extern "C" {
+
+const char* oz2_status_string(int status) {
+  switch (status) {
+    case OZ2_OK: return "OZ2_OK";
+    case OZ2_ERR_INVALID_ARG: return "OZ2_ERR_INVALID_ARG";
+    case OZ2_ERR_UNSUPPORTED_R: return "OZ2_ERR_UNSUPPORTED_R";
+    case OZ2_ERR_ALLOC: return "OZ2_ERR_ALLOC";
+    case OZ2_ERR_CUDA: return "OZ2_ERR_CUDA";
+    case OZ2_ERR_TIMEOUT: return "OZ2_ERR_TIMEOUT";
+    case OZ2_ERR_UNSUPPORTED: return "OZ2_ERR_UNSUPPORTED";
+    default: return "OZ2_ERR_UNKNOWN";
+  }
+}
+
+int oz2_plane_layout(int num_moduli, int32_t* plane_offset) {
+  if (num_moduli < 1 || num_moduli > kMaxModuli) return OZ2_ERR_UNSUPPORTED_R;
+  int p = 0;
+  for (int i = 0; i < num_moduli; ++i) {
+    if (plane_offset) plane_offset[i] = p;
+    p += isqrt_exact(kModuliAll[i]) ? 2 : 3;
+  }
+  return p;
+}
+
+size_t oz2_workspace_size(int64_t m, int64_t n, int64_t k, int num_moduli) {
+  if (m < 0 || n < 0 || k < 0 || num_moduli < 1 || num_moduli > kMaxModuli) return 0;
+  oz2_ws_layout L;
+  compute_layout(m, n, k, num_moduli, &L);
+  return L.total;
+}
+
+int oz2_workspace_layout(int64_t m, int64_t n, int64_t k, int num_moduli, oz2_ws_layout* out) {
+  if (!out || m < 0 || n < 0 || k < 0) return OZ2_ERR_INVALID_ARG;
+  if (num_moduli < 1 || num_moduli > kMaxModuli) return OZ2_ERR_UNSUPPORTED_R;
+  compute_layout(m, n, k, num_moduli, out);
+  return OZ2_OK;
+}
+
+int oz2_dgemm_ex(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, const double* B, int64_t ldb,
+                 double* C, int64_t ldc, int num_moduli, int quant, int scale, unsigned flags, void* workspace,
+                 size_t ws_bytes, void* stream) {
+  int st = check_sizes(m, n, k, lda, ldb, ldc);
+  if (st) return st;
+  if (num_moduli < 1 || num_moduli > kMaxModuli) return OZ2_ERR_UNSUPPORTED_R;
+  if ((quant != OZ2_QUANT_TZ && quant != OZ2_QUANT_RN) || (scale != OZ2_SCALE_R2 && scale != OZ2_SCALE_R1))
+    return OZ2_ERR_INVALID_ARG;
+  if (m == 0 || n == 0) return OZ2_OK;
+  if (!C || (k > 0 && (!A || !B))) return OZ2_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (k == 0) return to_status(cudaMemset2DAsync(C, ldc * sizeof(double), 0, m * sizeof(double), n, s));
+
+  oz2_ws_layout L;
+  compute_layout(m, n, k, num_moduli, &L);
+  if (!workspace || ws_bytes < L.total || (reinterpret_cast<uintptr_t>(workspace) & 255)) return OZ2_ERR_ALLOC;
+  DeviceState* ds = nullptr;
+  if ((st = device_state(&ds)) != OZ2_OK) return st;
+  const Oz2Moduli mods = build_moduli(num_moduli, quant);
+
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  int32_t* ra = reinterpret_cast<int32_t*>(ws + L.ra);
+  int32_t* cb = reinterpret_cast<int32_t*>(ws + L.cb);
+  uint8_t* rf = ws + L.row_flag;
+  uint8_t* cf = ws + L.col_flag;
+  int32_t* d = reinterpret_cast<int32_t*>(ws + L.d);
+  int32_t* e = reinterpret_cast<int32_t*>(ws + L.e);
+  float* urow = reinterpret_cast<float*>(ws + L.urow);
+  int* misc = reinterpret_cast<int*>(ws + L.misc);
+  uint8_t* mag_a = ws + L.mag_a;
+  uint8_t* mag_b = ws + L.mag_b;
+  uint8_t* pa = ws + L.planes_a;
+  uint8_t* pb = ws + L.planes_b;
+  int16_t* res = reinterpret_cast<int16_t*>(ws + L.residues);
+
+  const bool timing = (flags & OZ2_FLAG_TIMING) != 0;
+  const bool simt = (flags & OZ2_FLAG_DEBUG_SIMT_GEMM) != 0;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  HostStats& hs = g_host_stats[dev];
+  TimingSet* ts = nullptr;
+  if (timing) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    ts = &hs.sets[hs.next];
+    hs.next = (hs.next + 1) % kTimingSets;
+    harvest(hs, *ts);
+    if (!ts->created) {
+      for (int i = 0; i < 9; ++i) cudaEventCreate(&ts->ev[i]);
+      ts->created = true;
+    }
+  }
+  auto mark = [&](int i) {
+    if (ts) cudaEventRecord(ts->ev[i], s);
+  };
+
+  cudaError_t err = cudaSuccess;
+  count_launch();
+  reset_status_kernel<<<1, 1, 0, s>>>(ds->status);
+  mark(0);
+  if (err == cudaSuccess)
+    err = launch_scan(m, n, k, A, lda, B, ldb, flags, ScanOut{ra, cb, rf, cf}, ds->status, s);
+  mark(1);
+  if (scale == OZ2_SCALE_R2) {
+    if (err == cudaSuccess) err = cudaMemsetAsync(urow, 0, sizeof(float) * m, s);
+    if (err == cudaSuccess)
+      err = launch_magnitude_planes(m, n, k, A, lda, B, ldb, ra, cb, rf, cf, mag_a, mag_b, s);
+    mark(2);
+    if (err == cudaSuccess)
+      err = launch_plane_gemm(m, n, L.k_pad, mods, mag_a, mag_b, simt ? 3 : 1, nullptr, urow, ds->status, s);
+    mark(3);
+  } else {
+    mark(2);
+    mark(3);
+  }
+  if (err == cudaSuccess) err = launch_choose_scales(m, n, k, mods, scale, urow, ra, cb, rf, cf, d, e, ds->status, s);
+  mark(4);
+  if (err == cudaSuccess)
+    err = launch_deconstruct(m, n, k, mods, ds->table, A, lda, B, ldb, d, e, rf, cf, quant, pa, pb, s);
+  mark(5);
+  if (err == cudaSuccess)
+    err = launch_plane_gemm(m, n, L.k_pad, mods, pa, pb, simt ? 2 : 0, res, nullptr, ds->status, s);
+  mark(6);
+  if (err == cudaSuccess) err = launch_reconstruct(m, n, mods, res, m, d, e, C, ldc, s);
+  mark(7);
+  if (err == cudaSuccess) err = launch_fallback_lists(m, n, k, A, lda, B, ldb, rf, cf, misc, C, ldc, s);
+  mark(8);
+
+  hs.k_slab = static_cast<int>(std::min<int64_t>(kKSlab, L.k_pad));
+  if (ts) ts->pending = true;
+  return to_status(err);
+}
+
+int oz2_dgemm(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, const double* B, int64_t ldb,
+              double* C, int64_t ldc, int num_moduli, void* stream) {
+  int st = check_sizes(m, n, k, lda, ldb, ldc);
+  if (st) return st;
+  if (num_moduli < 1 || num_moduli > kMaxModuli) return OZ2_ERR_UNSUPPORTED_R;
+  if (m == 0 || n == 0 || k == 0)
+    return oz2_dgemm_ex(m, n, k, A, lda, B, ldb, C, ldc, num_moduli, OZ2_QUANT_TZ, OZ2_SCALE_R2, 0, nullptr, 0,
+                        stream);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  size_t bytes = oz2_workspace_size(m, n, k, num_moduli);
+  void* ws = nullptr;
+  if (cudaMallocAsync(&ws, bytes, s) != cudaSuccess) {
+    cudaGetLastError();
+    return OZ2_ERR_ALLOC;
+  }
+  st = oz2_dgemm_ex(m, n, k, A, lda, B, ldb, C, ldc, num_moduli, OZ2_QUANT_TZ, OZ2_SCALE_R2, 0, ws, bytes, stream);
+  cudaError_t e2 = cudaFreeAsync(ws, s);
+  if (st == OZ2_OK && e2 != cudaSuccess) st = OZ2_ERR_CUDA;
+  return st;
+}
+
+int oz2_dgemm_host(int64_t m, int64_t n, int64_t k, const double* hA, int64_t lda, const double* hB, int64_t ldb,
+                   double* hC, int64_t ldc, int num_moduli, void* stream) {
+  int st = check_sizes(m, n, k, lda, ldb, ldc);
+  if (st) return st;
+  if (num_moduli < 1 || num_moduli > kMaxModuli) return OZ2_ERR_UNSUPPORTED_R;
+  if (m == 0 || n == 0) return OZ2_OK;
+  if (!hC || (k > 0 && (!hA || !hB))) return OZ2_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const size_t bA = align256(sizeof(double) * m * k), bB = align256(sizeof(double) * k * n),
+               bC = align256(sizeof(double) * m * n);
+  const size_t ws = k > 0 ? oz2_workspace_size(m, n, k, num_moduli) : 0;
+  uint8_t* buf = nullptr;
+  if (cudaMallocAsync(reinterpret_cast<void**>(&buf), bA + bB + bC + ws, s) != cudaSuccess) {
+    cudaGetLastError();
+    return OZ2_ERR_ALLOC;
+  }
+  double* dA = reinterpret_cast<double*>(buf);
+  double* dB = reinterpret_cast<double*>(buf + bA);
+  double* dC = reinterpret_cast<double*>(buf + bA + bB);
+  cudaError_t err = cudaSuccess;
+  if (k > 0) {
+    err = cudaMemcpy2DAsync(dA, sizeof(double) * m, hA, sizeof(double) * lda, sizeof(double) * m, k,
+                            cudaMemcpyHostToDevice, s);
+    if (err == cudaSuccess)
+      err = cudaMemcpy2DAsync(dB, sizeof(double) * k, hB, sizeof(double) * ldb, sizeof(double) * k, n,
+                              cudaMemcpyHostToDevice, s);
+  }
+  if (err == cudaSuccess)
+    st = oz2_dgemm_ex(m, n, k, dA, m, dB, std::max<int64_t>(1, k), dC, m, num_moduli, OZ2_QUANT_TZ, OZ2_SCALE_R2,
+                      0, k > 0 ? buf + bA + bB + bC : nullptr, ws, stream);
+  if (err == cudaSuccess && st == OZ2_OK)
+    err = cudaMemcpy2DAsync(hC, sizeof(double) * ldc, dC, sizeof(double) * m, sizeof(double) * m, n,
+                            cudaMemcpyDeviceToHost, s);
+  cudaFreeAsync(buf, s);
+  if (cudaStreamSynchronize(s) != cudaSuccess && err == cudaSuccess) err = cudaErrorUnknown;
+  if (st != OZ2_OK) return st;
+  return to_status(err);
+}
+
+int oz2_get_stats(oz2_stats* out) {
+  if (!out) return OZ2_ERR_INVALID_ARG;
+  DeviceState* ds = nullptr;
+  int st = device_state(&ds);
+  if (st) return st;
+  if (cudaDeviceSynchronize() != cudaSuccess) return OZ2_ERR_CUDA;
+  Oz2Device h;
+  if (cudaMemcpy(&h, ds->status, sizeof(h), cudaMemcpyDeviceToHost) != cudaSuccess) return OZ2_ERR_CUDA;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  std::memset(out, 0, sizeof(*out));
+  out->status = h.status ? OZ2_ERR_TIMEOUT : OZ2_OK;
+  out->fallback_rows = h.fallback_rows;
+  out->fallback_cols = h.fallback_cols;
+  float u;
+  std::memcpy(&u, &h.u_max_bits, sizeof(u));
+  int ue = 0;
+  if (u > 0.f) {
+    unsigned b;
+    std::memcpy(&b, &u, sizeof(b));
+    ue = static_cast<int>((b >> 23) & 0xFF) - 127 + ((b & 0x7FFFFFu) ? 1 : 0);
+  }
+  out->u_max = ue;
+  out->s = h.s;
+  HostStats& hs = g_host_stats[dev];
+  {
+    std::lock_guard<std::mutex> lk(g_mu);
+    for (int i = 0; i < kTimingSets; ++i) harvest(hs, hs.sets[i]);
+    out->k_slab = hs.k_slab;
+    out->timed_calls = hs.timed;
+    for (int i = 0; i < 8; ++i) out->stage_ms[i] = hs.timed ? static_cast<float>(hs.stage_sum[i] / hs.timed) : 0.f;
+    for (int i = 0; i < 8; ++i) hs.stage_sum[i] = 0;
+    hs.timed = 0;
+  }
+  out->kernel_launches = g_launches.exchange(0);
+  return OZ2_OK;
+}
+
+int oz2_check_device_status(void) {
+  DeviceState* ds = nullptr;
+  int st = device_state(&ds);
+  if (st) return st;
+  if (cudaDeviceSynchronize() != cudaSuccess) return OZ2_ERR_CUDA;
+  int v = 0;
+  if (cudaMemcpy(&v, ds->status, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return OZ2_ERR_CUDA;
+  if (v) {
+    int zero = 0;
+    cudaMemcpy(ds->status, &zero, sizeof(int), cudaMemcpyHostToDevice);
+    return OZ2_ERR_TIMEOUT;
+  }
+  return OZ2_OK;
+}
+
+// ----------------------------- stage entry points ---------------------------
+int oz2_scan(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, const double* B, int64_t ldb,
+             unsigned flags, int32_t* ra, int32_t* cb, uint8_t* row_flag, uint8_t* col_flag, void* stream) {
+  int st = check_sizes(m, n, k, lda, ldb, std::max<int64_t>(1, m));
+  if (st) return st;
+  if ((m && (!ra || !row_flag)) || (n && (!cb || !col_flag)) || (k && m && !A) || (k && n && !B))
+    return OZ2_ERR_INVALID_ARG;
+  DeviceState* ds = nullptr;
+  if ((st = device_state(&ds)) != OZ2_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  count_launch();
+  reset_status_kernel<<<1, 1, 0, s>>>(ds->status);
+  return to_status(launch_scan(m, n, k, A, lda, B, ldb, flags, ScanOut{ra, cb, row_flag, col_flag}, ds->status, s));
+}
+
+int oz2_scale(int64_t m, int64_t n, int64_t k, int num_moduli, const double* A, int64_t lda, const double* B,
+              int64_t ldb, const int32_t* ra, const int32_t* cb, const uint8_t* row_flag, const uint8_t* col_flag,
+              int quant, int scale, uint8_t* mag_a, uint8_t* mag_b, float* urow, int32_t* d, int32_t* e,
+              void* stream) {
+  int st = check_sizes(m, n, k, lda, ldb, std::max<int64_t>(1, m));
+  if (st) return st;
+  if (num_moduli < 1 || num_moduli > kMaxModuli) return OZ2_ERR_UNSUPPORTED_R;
+  if (m == 0 || n == 0 || k == 0) return OZ2_ERR_INVALID_ARG;
+  if (!A || !B || !ra || !cb || !row_flag || !col_flag || !mag_a || !mag_b || !urow || !d || !e)
+    return OZ2_ERR_INVALID_ARG;
+  DeviceState* ds = nullptr;
+  if ((st = device_state(&ds)) != OZ2_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const Oz2Moduli mods = build_moduli(num_moduli, quant);
+  const int64_t k_pad = (k + kKPad - 1) / kKPad * kKPad;
+  count_launch();
+  reset_status_kernel<<<1, 1, 0, s>>>(ds->status);
+  cudaError_t err = cudaMemsetAsync(urow, 0, sizeof(float) * m, s);
+  if (scale == OZ2_SCALE_R2) {
+    if (err == cudaSuccess)
+      err = launch_magnitude_planes(m, n, k, A, lda, B, ldb, ra, cb, row_flag, col_flag, mag_a, mag_b, s);
+    if (err == cudaSuccess) err = launch_plane_gemm(m, n, k_pad, mods, mag_a, mag_b, 1, nullptr, urow, ds->status, s);
+  }
+  if (err == cudaSuccess)
+    err = launch_choose_scales(m, n, k, mods, scale, urow, ra, cb, row_flag, col_flag, d, e, ds->status, s);
+  return to_status(err);
+}
+
+int oz2_deconstruct(int64_t m, int64_t n, int64_t k, int num_moduli, const double* A, int64_t lda, const double* B,
+                    int64_t ldb, const int32_t* d, const int32_t* e, const uint8_t* row_flag, const uint8_t* col_flag,
+                    int quant, uint8_t* planes_a, uint8_t* planes_b, void* stream) {
+  int st = check_sizes(m, n, k, lda, ldb, std::max<int64_t>(1, m));
+  if (st) return st;
+  if (num_moduli < 1 || num_moduli > kMaxModuli) return OZ2_ERR_UNSUPPORTED_R;
+  if (k == 0 || !A || !B || !d || !e || !row_flag || !col_flag || !planes_a || !planes_b) return OZ2_ERR_INVALID_ARG;
+  DeviceState* ds = nullptr;
+  if ((st = device_state(&ds)) != OZ2_OK) return st;
+  const Oz2Moduli mods = build_moduli(num_moduli, quant);
+  return to_status(launch_deconstruct(m, n, k, mods, ds->table, A, lda, B, ldb, d, e, row_flag, col_flag, quant,
+                                      planes_a, planes_b, static_cast<cudaStream_t>(stream)));
+}
+
+int oz2_residue_gemm(int64_t m, int64_t n, int64_t k, int num_moduli, const uint8_t* planes_a,
+                     const uint8_t* planes_b, int16_t* residues, void* stream) {
+  if (m <= 0 || n <= 0 || k <= 0 || !planes_a || !planes_b || !residues) return OZ2_ERR_INVALID_ARG;
+  if (num_moduli < 1 || num_moduli > kMaxModuli) return OZ2_ERR_UNSUPPORTED_R;
+  if (m >= (1LL << 31) || n >= (1LL << 31) || k > (1LL << 24)) return OZ2_ERR_UNSUPPORTED;
+  DeviceState* ds = nullptr;
+  int st = device_state(&ds);
+  if (st) return st;
+  const Oz2Moduli mods = build_moduli(num_moduli, OZ2_QUANT_TZ);
+  const int64_t k_pad = (k + kKPad - 1) / kKPad * kKPad;
+  return to_status(launch_plane_gemm(m, n, k_pad, mods, planes_a, planes_b, 0, residues, nullptr, ds->status,
+                                     static_cast<cudaStream_t>(stream)));
+}
+
+int oz2_residue_gemm_simt(int64_t m, int64_t n, int64_t k, int num_moduli, const uint8_t* planes_a,
+                          const uint8_t* planes_b, int16_t* residues, void* stream) {
+  if (m <= 0 || n <= 0 || k <= 0 || !planes_a || !planes_b || !residues) return OZ2_ERR_INVALID_ARG;
+  if (num_moduli < 1 || num_moduli > kMaxModuli) return OZ2_ERR_UNSUPPORTED_R;
+  DeviceState* ds = nullptr;
+  int st = device_state(&ds);
+  if (st) return st;
+  const Oz2Moduli mods = build_moduli(num_moduli, OZ2_QUANT_TZ);
+  const int64_t k_pad = (k + kKPad - 1) / kKPad * kKPad;
+  return to_status(launch_plane_gemm(m, n, k_pad, mods, planes_a, planes_b, 2, residues, nullptr, ds->status,
+                                     static_cast<cudaStream_t>(stream)));
+}
+
+int oz2_reconstruct(int64_t m, int64_t n, int num_moduli, const int16_t* residues, int64_t ldr, const int32_t* d,
+                    const int32_t* e, double* C, int64_t ldc, void* stream) {
+  if (m < 0 || n < 0 || ldr < std::max<int64_t>(1, m) || ldc < std::max<int64_t>(1, m)) return OZ2_ERR_INVALID_ARG;
+  if (num_moduli < 1 || num_moduli > kMaxModuli) return OZ2_ERR_UNSUPPORTED_R;
+  if (m && n && (!residues || !d || !e || !C)) return OZ2_ERR_INVALID_ARG;
+  const Oz2Moduli mods = build_moduli(num_moduli, OZ2_QUANT_TZ);
+  return to_status(launch_reconstruct(m, n, mods, residues, ldr, d, e, C, ldc, static_cast<cudaStream_t>(stream)));
+}
+
+int oz2_fallback(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, const double* B, int64_t ldb,
+                 const uint8_t* row_flag, const uint8_t* col_flag, double* C, int64_t ldc, void* stream) {
+  int st = check_sizes(m, n, k, lda, ldb, ldc);
+  if (st) return st;
+  if (m == 0 || n == 0) return OZ2_OK;
+  if (!row_flag || !col_flag || !C || (k && (!A || !B))) return OZ2_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int* scratch = nullptr;
+  if (cudaMallocAsync(reinterpret_cast<void**>(&scratch), sizeof(int) * (m + n + 2), s) != cudaSuccess) {
+    cudaGetLastError();
+    return OZ2_ERR_ALLOC;
+  }
+  cudaError_t err = launch_fallback_lists(m, n, k, A, lda, B, ldb, row_flag, col_flag, scratch, C, ldc, s);
+  cudaFreeAsync(scratch, s);
+  return to_status(err);
+}
+
+int oz2_native_dgemm(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, const double* B, int64_t ldb,
+                     double* C, int64_t ldc, void* stream) {
+  int st = check_sizes(m, n, k, lda, ldb, ldc);
+  if (st) return st;
+  if (m == 0 || n == 0) return OZ2_OK;
+  if (!C || (k && (!A || !B))) return OZ2_ERR_INVALID_ARG;
+  return to_status(launch_native(m, n, k, A, lda, B, ldb, C, ldc, static_cast<cudaStream_t>(stream)));
+}
+
+}  // extern "C"

@@ -1,0 +1,255 @@
+// Internal definitions shared by the liboz2 translation units.
+//
+// Modulus constants are computed once per r on the host (oz2_api.cu) and
+// passed to kernels by value (__grid_constant__), so concurrent calls with
+// different r never share mutable constant memory.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/oz2.h"
+
+namespace oz2 {
+
+constexpr int kMaxModuli = 16;
+constexpr int kMaxPlanes = 48;         // 3 per modulus at most
+constexpr int kKPad = 128;             // k is padded to a multiple of this
+constexpr int kMagClampMax = 9;        // 2^-9: smallest E4M3 magnitude
+constexpr int kFallbackWindow = 128;   // binades from the median (fallback)
+// Exact FP32 accumulation (Eq. accum-exact): every accumulator term is at
+// most 512 in magnitude (square cross term d1e0 + d0e1; nonsquare terms are
+// ≤ 484), so K_slab · 512 ≤ 2^24 holds for K_slab = 32768.
+constexpr int kKSlab = 32768;
+
+// Device status word values (stored in Oz2Device::status).
+constexpr int kStatusTimeout = 1;
+
+struct Oz2Moduli {
+  int r;
+  int nplanes;
+  int T;                        // range exponent of the scale choice
+  int m[kMaxModuli];
+  int sq_base[kMaxModuli];      // s for m = s², 0 for nonsquare
+  int plane_off[kMaxModuli];    // first plane of modulus i
+  int table_off[kMaxModuli];    // first entry of modulus i in the plane table
+  uint32_t magic[kMaxModuli];   // ⌈2^(32+sh)/m⌉, sh = ⌊log2(m-1)⌋
+  int magic_sh[kMaxModuli];
+  int limb[kMaxModuli][4];      // 2^(16j) mod m
+  int negoff[kMaxModuli];       // multiple of m ≥ 2^28 (sign handling)
+  // Garner (Eq. garner): pmod[k][j] = (m_0 ⋯ m_{j-1}) mod m_k for j < k,
+  // inv[k] = (m_0 ⋯ m_{k-1})^-1 mod m_k, goff[k] = multiple of m_k ≥ 2^27.
+  int pmod[kMaxModuli][kMaxModuli];
+  int inv[kMaxModuli];
+  int goff[kMaxModuli];
+  // M and ⌈M/2⌉ as 3×64-bit little-endian limbs.
+  unsigned long long M[3];
+  unsigned long long Mhalf[3];
+  int table_entries;            // Σ m_i
+};
+
+// Per-device status block (in device global memory, owned by oz2_api.cu).
+struct Oz2Device {
+  int status;                   // 0, or kStatusTimeout (sticky until read)
+  int timeout_site;
+  int fallback_rows;
+  int fallback_cols;
+  int u_max_bits;               // float bits of max_ij U_ij ("+1" pass)
+  int s;                        // column budget (R2) or pB (R1)
+  int pad[10];
+};
+
+// Residue of y (< 2^31) modulo m with a precomputed multiplier
+// (Granlund & Montgomery 1994, "Division by invariant integers using
+// multiplication"): q = ⌊y·magic / 2^(32+sh)⌋ = ⌊y/m⌋ because the error
+// e = magic·m - 2^(32+sh) < m and y·e < 2^(32+sh) for y < 2^31.
+__device__ __forceinline__ uint32_t mod_magic(uint32_t y, uint32_t m, uint32_t magic, int sh) {
+  uint32_t q = __umulhi(y, magic) >> sh;
+  return y - q * m;
+}
+
+// ---------------------------------------------------------------------------
+// PTX wrappers (sm_100-family tcgen05 / TMA / mbarrier), with bounded waits.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count));
+}
+
+__device__ __forceinline__ void fence_barrier_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n"
+      " mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Wait for the given phase parity; gives up after ~`limit` clock cycles and
+// returns false.  Every spin in the library goes through this.
+__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity, long long limit) {
+  if (mbar_try_wait(bar, parity)) return true;
+  long long t0 = clock64();
+  for (uint32_t it = 1;; ++it) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((it & 255u) == 0 && clock64() - t0 > limit) return false;
+  }
+}
+
+// 3-D tiled TMA load into shared memory, completing on an mbarrier.
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map, uint32_t bar,
+                                           int x, int y, int z) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(x), "r"(y), "r"(z)
+      : "memory");
+}
+
+__device__ __forceinline__ void prefetch_tensormap(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
+// --- tcgen05 -----------------------------------------------------------------
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem),
+               "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// D[tmem] (+)= A[smem] · B[smem]^T, kind::f8f6f4, issued by one thread.
+__device__ __forceinline__ void mma_f8(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                       uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrive on an mbarrier once all prior tcgen05 ops of this thread complete.
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+      : "memory");
+}
+
+// 32 lanes × 32 bits, 32 consecutive columns per thread.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
+        "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]),
+        "=r"(v[14]), "=r"(v[15]), "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]),
+        "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]), "=r"(v[25]),
+        "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_ld_wait() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor for a K-major operand tile stored with the
+// 128-byte swizzle that TMA writes (rows of 128 bytes, 8-row atoms of 1024
+// bytes): start address >> 4 in bits [0,14), leading-byte offset (unused for
+// swizzled K-major, set to 1) in [16,30), stride-byte offset 1024 >> 4 in
+// [32,46), descriptor version 1 in [46,48), layout SWIZZLE_128B (2) in [61,64).
+__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr >> 4) & 0x3FFFu);
+  d |= static_cast<uint64_t>(1u) << 16;
+  d |= static_cast<uint64_t>(1024u >> 4) << 32;
+  d |= static_cast<uint64_t>(1u) << 46;
+  d |= static_cast<uint64_t>(2u) << 61;
+  return d;
+}
+
+// Instruction descriptor, kind::f8f6f4: D = F32 (bits 4-5 = 1), A = B = E4M3
+// (bits 7-9, 10-12 = 0), both K-major (bits 15, 16 = 0), N >> 3 in bits
+// 17-22, M >> 4 in bits 24-28.
+__host__ __device__ constexpr uint32_t idesc_f8_f32(int M, int N) {
+  return (1u << 4) | (static_cast<uint32_t>(N >> 3) << 17) | (static_cast<uint32_t>(M >> 4) << 24);
+}
+
+}  // namespace oz2
+
+// Host-side launchers (defined in the kernel translation units).
+namespace oz2 {
+// Counts kernel launches made by the library (read through oz2_get_stats).
+void count_launch(int n = 1);
+struct ScanOut {
+  int32_t* ra;
+  int32_t* cb;
+  uint8_t* row_flag;
+  uint8_t* col_flag;
+};
+cudaError_t launch_scan(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda,
+                        const double* B, int64_t ldb, unsigned flags, ScanOut out,
+                        Oz2Device* dev, cudaStream_t st);
+cudaError_t launch_magnitude_planes(int64_t m, int64_t n, int64_t k, const double* A,
+                                    int64_t lda, const double* B, int64_t ldb, const int32_t* ra,
+                                    const int32_t* cb, const uint8_t* row_flag,
+                                    const uint8_t* col_flag, uint8_t* mag_a, uint8_t* mag_b,
+                                    cudaStream_t st);
+cudaError_t launch_choose_scales(int64_t m, int64_t n, int64_t k, const Oz2Moduli& mods,
+                                 int scale_mode, const float* urow, const int32_t* ra,
+                                 const int32_t* cb, const uint8_t* row_flag,
+                                 const uint8_t* col_flag, int32_t* d, int32_t* e,
+                                 Oz2Device* dev, cudaStream_t st);
+cudaError_t launch_deconstruct(int64_t m, int64_t n, int64_t k, const Oz2Moduli& mods,
+                               const uint32_t* table, const double* A, int64_t lda,
+                               const double* B, int64_t ldb, const int32_t* d, const int32_t* e,
+                               const uint8_t* row_flag, const uint8_t* col_flag, int quant,
+                               uint8_t* planes_a, uint8_t* planes_b, cudaStream_t st);
+cudaError_t launch_plane_gemm(int64_t m, int64_t n, int64_t k_pad, const Oz2Moduli& mods,
+                              const uint8_t* planes_a, const uint8_t* planes_b, int mode,
+                              int16_t* residues, float* urow, Oz2Device* dev, cudaStream_t st);
+cudaError_t launch_reconstruct(int64_t m, int64_t n, const Oz2Moduli& mods,
+                               const int16_t* residues, int64_t ldr, const int32_t* d,
+                               const int32_t* e, double* C, int64_t ldc, cudaStream_t st);
+cudaError_t launch_fallback_lists(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda,
+                                  const double* B, int64_t ldb, const uint8_t* row_flag,
+                                  const uint8_t* col_flag, int* scratch, double* C, int64_t ldc,
+                                  cudaStream_t st);
+cudaError_t launch_native(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda,
+                          const double* B, int64_t ldb, double* C, int64_t ldc, cudaStream_t st);
+}  // namespace oz2

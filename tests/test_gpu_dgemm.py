@@ -1,0 +1,145 @@
+"""End-to-end parity of oz2_dgemm / oz2_dgemm_ex with the CPU oracle.
+
+Small and ragged shapes compare every entry bit-for-bit, along with the
+intermediates left in the workspace.  The 4096³ workload that bench.py times
+is checked in the same launch configuration: full scale vectors and a
+sample of rows of C, bit-exact.
+"""
+import numpy as np
+import pytest
+
+import workloads as wl
+from helpers import ensure_built, to_dev
+from oracle import cref
+from oracle import ozaki2 as orc
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def oz():
+    ensure_built()
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2606_06510_gb300 as oz
+    oz.lib()
+    return oz
+
+
+def run_ex(oz, A, B, r, quant="tz", scale="r2", flags=0):
+    C, ws = oz.oz2_dgemm_ex(to_dev(A), to_dev(B), num_moduli=r, quant=quant, scale=scale, flags=flags)
+    views = oz.workspace_views(ws, A.shape[0], B.shape[1], A.shape[1], r)
+    assert oz.oz2_check_device_status() == 0
+    return C.cpu().numpy(), {k: v.cpu().numpy() for k, v in views.items()}
+
+
+def assert_same(got, want):
+    same = (got == want) | (np.isnan(got) & np.isnan(want))
+    if not same.all():
+        bad = np.argwhere(~same)
+        i, j = bad[0]
+        raise AssertionError(f"{len(bad)} entries differ; first ({i},{j}): {got[i, j]!r} vs {want[i, j]!r}")
+    assert np.array_equal(np.signbit(got[~np.isnan(got)]), np.signbit(want[~np.isnan(want)]))
+
+
+def test_small_workload_bit_exact_and_accurate(oz):
+    A, B = wl.make_inputs(wl.WORKLOADS["dgemm_256"])
+    res = orc.oz2_dgemm(A, B, 12)
+    C, v = run_ex(oz, A, B, 12)
+    assert_same(C, res.C)
+    assert np.array_equal(v["d"], res.d) and np.array_equal(v["e"], res.e)
+    assert np.array_equal(v["residues"].transpose(0, 2, 1), res.residues)
+    assert cref.scaled_error(C, A, B) <= 1e-15
+    # the production entry (own workspace) gives the same bits
+    C2 = oz.oz2_dgemm(to_dev(A), to_dev(B), num_moduli=12).cpu().numpy()
+    assert_same(C2, res.C)
+
+
+@pytest.mark.parametrize("shape", [(1, 1, 1), (100, 77, 333), (257, 129, 129), (64, 300, 7), (3, 5, 1000)])
+def test_ragged_shapes(oz, shape):
+    m, n, k = shape
+    A = wl.random_matrix(m, k, 1.0, m + n)
+    B = wl.random_matrix(k, n, 1.0, k)
+    res = orc.oz2_dgemm(A, B, 12)
+    C, _ = run_ex(oz, A, B, 12)
+    assert_same(C, res.C)
+
+
+@pytest.mark.parametrize("r", [1, 2, 6, 11, 12, 13, 16])
+def test_moduli_counts(oz, r):
+    A, B = wl.random_matrix(64, 160, 0.5, 1), wl.random_matrix(160, 48, 0.5, 2)
+    res = orc.oz2_dgemm(A, B, r)
+    C, v = run_ex(oz, A, B, r)
+    assert_same(C, res.C)
+    assert np.array_equal(v["residues"].transpose(0, 2, 1), res.residues)
+
+
+@pytest.mark.parametrize("quant", ["tz", "rn"])
+@pytest.mark.parametrize("scale", ["r2", "r1"])
+def test_variants(oz, quant, scale):
+    A, B = wl.random_matrix(96, 200, 2.0, 5), wl.random_matrix(200, 80, 2.0, 6)
+    res = orc.oz2_dgemm(A, B, 12, quant=quant, scale=scale)
+    C, _ = run_ex(oz, A, B, 12, quant=quant, scale=scale)
+    assert_same(C, res.C)
+
+
+def test_simt_diagnostic_engine_matches(oz):
+    A, B = wl.random_matrix(130, 140, 1.0, 8), wl.random_matrix(140, 70, 1.0, 9)
+    res = orc.oz2_dgemm(A, B, 12)
+    C, _ = run_ex(oz, A, B, 12, flags=oz.FLAG_DEBUG_SIMT_GEMM)
+    assert_same(C, res.C)
+
+
+def test_fallback_and_special_values(oz):
+    A = np.array(wl.random_matrix(150, 90, 1.0, 11), order="F")
+    B = np.array(wl.random_matrix(90, 70, 1.0, 12), order="F")
+    A[3, :] *= 2.0 ** 300
+    A[8, :] *= 2.0 ** -300
+    A[20, 4] = np.nan
+    A[21, 5] = -np.inf
+    A[30, :] = 0.0
+    A[31, :] *= 2.0 ** -1060
+    B[7, 9] = np.inf
+    B[:, 12] = 0.0
+    res = orc.oz2_dgemm(A, B, 12)
+    C, v = run_ex(oz, A, B, 12)
+    assert_same(C, res.C)
+    st = oz.oz2_get_stats()
+    # rows 3, 8 (2^±300), 20, 21 (non-finite) and 31 (2^-1060: far below the median)
+    assert st["fallback_rows"] == int(res.row_flag.sum()) == 5
+    assert st["fallback_cols"] == int(res.col_flag.sum()) == 1
+    assert np.array_equal(v["row_flag"] & 1, res.row_flag.astype(np.uint8))
+
+
+def test_zero_and_empty(oz):
+    import torch
+    A = np.zeros((50, 40))
+    B = wl.random_matrix(40, 30, 0.5, 1)
+    C, _ = run_ex(oz, A, B, 12)
+    assert np.all(C == 0) and not np.signbit(C).any()
+    # k = 0: C = 0
+    Cd = to_dev(np.full((5, 6), 3.0))
+    oz.oz2_dgemm(torch.empty((5, 0), dtype=torch.float64, device="cuda"),
+                 torch.empty((0, 6), dtype=torch.float64, device="cuda"), C=Cd)
+    assert np.all(Cd.cpu().numpy() == 0)
+
+
+def test_integer_inputs_exact(oz):
+    rng = np.random.default_rng(3)
+    A = rng.integers(-2**20, 2**20, size=(70, 90)).astype(np.float64)
+    B = rng.integers(-2**20, 2**20, size=(90, 50)).astype(np.float64)
+    C, _ = run_ex(oz, A, B, 12)
+    assert np.array_equal(C, A @ B)
+
+
+def test_bench_workload_full_size_sampled(oz):
+    """4096³, r = 12, φ = 0.5: the configuration bench.py times."""
+    w = wl.WORKLOADS["dgemm_4096"]
+    A, B = wl.make_inputs(w)
+    rows = np.array([0, 1, 127, 128, 2048, 4000, 4095])
+    res = orc.oz2_dgemm(A, B, w.r, rows=rows)
+    C, v = run_ex(oz, A, B, w.r)
+    assert np.array_equal(v["d"], res.d) and np.array_equal(v["e"], res.e)
+    assert_same(C[rows], res.C)
+    assert cref.scaled_error(C, A, B, rows=rows[:3]) <= 1e-15
