@@ -18,6 +18,7 @@ bounded sample of the same workload and metric.
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import os
 import statistics
@@ -35,6 +36,23 @@ import workloads as wl  # noqa: E402
 METRIC = "effective FP64 TFLOPS (2mnk/s) and % of FP8 tensor peak/alpha, per moduli count"
 L2_BYTES = 126 * 2**20
 FP8_TO_BF16 = 2.0   # nominal dense FP8 / BF16 tensor ratio (4.5 / 2.25 PFLOP/s)
+GEMM_SOURCE = os.path.join(ROOT, "paper_2606_06510_gb300", "csrc", "k_gemm.cu")
+# DRAM read+write bytes of one residue-GEMM launch, from the ncu capture in
+# profiles/residue_gemm_dgemm_4096.md; reported only while the kernel source
+# is the one the counters were taken on.
+GEMM_TRAFFIC = {"workload": "dgemm_4096", "num_moduli": 12, "bytes": 4.505e9,
+                "sha256": "1456b7d158eb027f05dbb4ff283d4817fbfadfe04106d654887530d6e5dbde05"}
+
+
+def gemm_traffic(w, r):
+    try:
+        sha = hashlib.sha256(open(GEMM_SOURCE, "rb").read()).hexdigest()
+    except OSError:
+        return None
+    t = GEMM_TRAFFIC
+    if sha == t["sha256"] and w.name == t["workload"] and r == t["num_moduli"]:
+        return t["bytes"]
+    return None
 
 
 def parse():
@@ -215,7 +233,7 @@ def run_oz2(args):
     gemm_flops = work["residue_gemm"][1]
     achieved = gemm_flops / (gemm_ms * 1e-3) / 1e12
     roofline = {"bound": "tensor", "achieved": round(achieved, 1), "peak": round(fp8_peak, 1), "unit": "TFLOP/s",
-                "frac": round(achieved / fp8_peak, 4), "traffic": None,
+                "frac": round(achieved / fp8_peak, 4), "traffic": gemm_traffic(w, r),
                 "kernel": "plane_gemm_tc_kernel<0> (residue GEMM, 3r FP8 plane products)",
                 "peak_source": f"{pk['source']} bf16 sustained x {FP8_TO_BF16} (nominal FP8/BF16 ratio)"}
 
