@@ -111,6 +111,26 @@ int oz2_dgemm_host(int64_t m, int64_t n, int64_t k,
                    double* h_C, int64_t ldc,
                    int num_moduli, void* stream);
 
+/* As oz2_dgemm, for callers that must not allocate device memory (a host
+ * framework whose allocator owns all device memory, code that may not block
+ * or fail on an allocation at run time, plug-ins handed only their input and
+ * output buffers).  The paper has no counterpart: this is a deployment
+ * variant of the same computation.  Instead of allocating a workspace it uses
+ * a fixed 32 MiB array in the library's own device memory (held on every GPU
+ * that loads the library until the process exits); problems whose
+ * oz2_workspace_size exceeds 32 MiB (about 512³ at num_moduli = 16) return
+ * OZ2_ERR_UNSUPPORTED.  It calls no allocation routine.  The first call on
+ * each device looks up the array's device address and uploads the library's
+ * digit-plane table; make that first call before any stream capture.  All
+ * calls share the one array: calls whose work overlaps on the GPU (different
+ * streams, or concurrent host threads) race and must be serialised by the
+ * caller.  Each call clears what it needs before using it. */
+int oz2_dgemm_noalloc(int64_t m, int64_t n, int64_t k,
+                      const double* d_A, int64_t lda,
+                      const double* d_B, int64_t ldb,
+                      double* d_C, int64_t ldc,
+                      int num_moduli, void* stream);
+
 /* Bytes of device workspace oz2_dgemm_ex needs for this problem. */
 size_t oz2_workspace_size(int64_t m, int64_t n, int64_t k, int num_moduli);
 

@@ -55,6 +55,7 @@ _SIGS = {
     "oz2_dgemm": (_I, [_I64, _I64, _I64, _P, _I64, _P, _I64, _P, _I64, _I, _P]),
     "oz2_workspace_size": (_SZ, [_I64, _I64, _I64, _I]),
     "oz2_dgemm_host": (_I, [_I64, _I64, _I64, _P, _I64, _P, _I64, _P, _I64, _I, _P]),
+    "oz2_dgemm_noalloc": (_I, [_I64, _I64, _I64, _P, _I64, _P, _I64, _P, _I64, _I, _P]),
     "oz2_dgemm_ex": (_I, [_I64, _I64, _I64, _P, _I64, _P, _I64, _P, _I64, _I, _I, _I, _U, _P, _SZ, _P]),
     "oz2_workspace_layout": (_I, [_I64, _I64, _I64, _I, ctypes.POINTER(oz2_ws_layout)]),
     "oz2_plane_layout": (_I, [_I, _P]),
