@@ -170,8 +170,10 @@ int oz2_workspace_layout(int64_t m, int64_t n, int64_t k, int num_moduli,
  * for B) every plane is a rows×k_pad byte matrix, row-major (k contiguous),
  * zero-padded from k to k_pad; plane p starts at byte p·rows·k_pad.  The
  * planes of modulus i are consecutive, starting at plane_offset[i]:
- *   square m_i = s²:  (d0, d1)            d = d0 + s·d1, balanced base s
- *   nonsquare:        (d0+d1, d0, d1)     d = d0 + 16·d1, carry-corrected
+ *   square m_i = s²:  (d0, d1)              d = d0 + s·d1, balanced base s
+ *   nonsquare, B:     (d0+d1, d0, d1)       d = d0 + 16·d1, carry-corrected
+ *   nonsquare, A:     (d0+d1, d0, -16·d1)   (pre-scaled for the merged
+ *                                           accumulator d0e0 - 16·d1e1, §2.5)
  * where d is the centred residue of the integer Ã (or B̃) entry.  Each byte
  * is the E4M3 code of the integer digit.  Writes num_moduli offsets and
  * returns the total plane count. */
@@ -227,8 +229,9 @@ int oz2_deconstruct(int64_t m, int64_t n, int64_t k, int num_moduli,
 /* Stage 4 (Eq. modgemm, Eq. sq-shortcut, Eq. kar): from digit planes in
  * the oz2_plane_layout order (k_pad = k rounded up to 128), the residue
  * matrices C^(i) = (A^(i) B^(i)) mod m_i, centred, r × (m×n column-major,
- * ld = m) int16.  Three FP8 tcgen05 MMAs per modulus with exact FP32
- * accumulation (Eq. accum-exact), reduced mod m_i every K-slab. */
+ * ld = m) int16.  Three FP8 tcgen05 MMAs per modulus into two FP32
+ * accumulators with exact accumulation (Eq. accum-exact), reduced mod m_i
+ * every K-slab (32768 for square moduli, 4096 for nonsquare ones). */
 int oz2_residue_gemm(int64_t m, int64_t n, int64_t k, int num_moduli,
                      const uint8_t* d_planes_a, const uint8_t* d_planes_b,
                      int16_t* d_residues, void* stream);

@@ -216,7 +216,7 @@ cudaError_t launch_magnitude_planes(int64_t m, int64_t n, int64_t k, const doubl
 }
 
 cudaError_t launch_deconstruct(int64_t m, int64_t n, int64_t k, const Oz2Moduli& mods,
-                               const uint32_t* table, const double* A, int64_t lda,
+                               const uint32_t* table_a, const uint32_t* table_b, const double* A, int64_t lda,
                                const double* B, int64_t ldb, const int32_t* d, const int32_t* e,
                                const uint8_t* row_flag, const uint8_t* col_flag, int quant,
                                uint8_t* planes_a, uint8_t* planes_b, cudaStream_t st) {
@@ -229,12 +229,12 @@ cudaError_t launch_deconstruct(int64_t m, int64_t n, int64_t k, const Oz2Moduli&
   if (m > 0) {
     OperandView va{A, 1, lda, m, d, row_flag, planes_a};
     count_launch();
-    planes_kernel<1><<<grid_for(m, k_pad), kDecThreads, smem, st>>>(va, k, k_pad, 0, rn, mods, table);
+    planes_kernel<1><<<grid_for(m, k_pad), kDecThreads, smem, st>>>(va, k, k_pad, 0, rn, mods, table_a);
   }
   if (n > 0) {
     OperandView vb{B, ldb, 1, n, e, col_flag, planes_b};
     count_launch();
-    planes_kernel<1><<<grid_for(n, k_pad), kDecThreads, smem, st>>>(vb, k, k_pad, 0, rn, mods, table);
+    planes_kernel<1><<<grid_for(n, k_pad), kDecThreads, smem, st>>>(vb, k, k_pad, 0, rn, mods, table_b);
   }
   return cudaGetLastError();
 }

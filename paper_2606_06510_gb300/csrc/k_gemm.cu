@@ -1,45 +1,49 @@
 // Phase 2 of Ozaki Scheme II on FP8 tensor cores (§2.3 Eq. modgemm; §2.5
 // Eq. sq-shortcut, Eq. kar, Eq. accum-exact) and the "+1" magnitude GEMM of
-// §2.4, as one tcgen05 kernel for sm_103a.
+// §2.4, as one persistent tcgen05 kernel for sm_103a running on CTA pairs.
 //
-// Per 128×128 output tile the kernel walks the moduli; per modulus it walks
-// k in steps of 128 bytes (four K=32 MMAs), loading the modulus's plane
-// tiles of A and B by TMA into shared memory and issuing three plane-product
-// MMAs per K=32 step into FP32 accumulators in tensor memory:
-//   square m = s²:  acc0 += d0·e0,  acc1 += d1·e0 + d0·e1
-//   nonsquare:      acc0 += (d0+d1)(e0+e1), acc1 += d0·e0, acc2 += d1·e1
-// Every K-slab (≤ 32768, Eq. accum-exact: all terms ≤ 512 so partial sums
-// stay exact integers below 2^24) the epilogue warps read the accumulators,
-// recombine them with the coefficients of Eq. sq-shortcut / Eq. kar, reduce
-// mod m and store the centred residue as int16 (adding the previous slab's).
+// Work unit = (modulus, 256×256 output tile); units are taken modulus-major
+// so that the planes of one modulus stay in L2 while every pair works on it.
+// A pair (cluster of 2 CTAs) computes its tile with cta_group::2 MMAs of
+// M = N = 256, K = 32: each CTA holds 128 rows of the A plane tile and 128
+// rows of the B plane tile in its own shared memory, and 128 rows × 256
+// columns of each FP32 accumulator in its tensor memory.
 //
-// Warp roles (192 threads): warp 0 = TMA producer, warp 1 = TMEM owner and
-// MMA issuer, warps 2..5 = epilogue (warp w reads TMEM lanes 32·(w mod 4)).
-// Every wait is bounded; on expiry the kernel records OZ2_ERR_TIMEOUT in the
-// device status word and all roles drain and exit.
+// Per modulus the three plane products of §2.5 accumulate into two TMEM
+// accumulators (256 columns each):
+//   square m = s²  : acc0 += d0·e0,            acc1 += d1·e0 + d0·e1
+//   nonsquare m    : acc0 += (d0+d1)(e0+e1),   acc1 += d0·e0 + (-16 d1)·e1
+// (the A operand stores its last nonsquare plane pre-scaled by -2^b, the
+// accumulator merge of §2.5 "Accumulators").  Every K-slab (32768 squares,
+// 4096 nonsquare: Eq. accum-exact) the epilogue reads the accumulators and
+// forms  v = acc0 + s·acc1  or  v = 16·acc0 - 15·acc1  mod m, adds the
+// previous slab's residue and stores the centred residue as int16.
+//
+// Pipeline: a stage is one (A plane, B plane) pair of 128-byte-deep tiles
+// (32 KiB per CTA), six stages.  Warp 0 of each CTA issues its CTA's TMA
+// loads, completing on the leader's stage barrier; warp 1 of the leader
+// issues the MMAs and multicasts stage releases and accumulator-ready
+// signals to both CTAs; warps 2..9 of both CTAs run the epilogue and release
+// the accumulators to the leader.  Every wait is bounded; on expiry the
+// kernel records OZ2_ERR_TIMEOUT in the device status word and drains.
+#include <algorithm>
+
 #include "oz2_common.cuh"
 
 namespace oz2 {
 
-constexpr int kBM = 128, kBN = 128, kBK = 128;   // tile rows, cols, k-bytes per step
-constexpr int kTileBytes = kBM * kBK;            // 16 KiB per plane tile (A and B alike)
-constexpr int kGemmThreads = 192;
+constexpr int kTileM = 256, kTileN = 256;        // per CTA pair
+constexpr int kRows = 128;                       // rows of A and of B per CTA
+constexpr int kBK = 128;                         // k-bytes per stage
+constexpr int kTileBytes = kRows * kBK;          // 16 KiB
+constexpr int kStageBytes = 2 * kTileBytes;      // A tile + B tile
+constexpr int kStages = 6;
+constexpr int kGemmThreads = 320;                // 10 warps
+constexpr int kEpiWarps = 8;
+constexpr int kTmemCols = 512;
+constexpr int kAccCols = 256;
+constexpr int kGroupM = 8;                       // tile rasterisation group
 constexpr long long kWaitLimit = 4000000000LL;   // ≈2 s at 2 GHz
-
-template <int MODE>
-struct GemmCfg;
-template <>
-struct GemmCfg<0> {                 // residue planes: ≤3 A and ≤3 B tiles per step
-  static constexpr int kStages = 2;
-  static constexpr int kMaxP = 3;
-  static constexpr int kTmemCols = 512;
-};
-template <>
-struct GemmCfg<1> {                 // magnitude plane ("+1" pass)
-  static constexpr int kStages = 4;
-  static constexpr int kMaxP = 1;
-  static constexpr int kTmemCols = 128;
-};
 
 // ---- epilogue arithmetic shared by the tensor-core and SIMT kernels --------
 // x - m·rint(x/m) for an exactly represented integer |x| < 2^24: the FMA
@@ -58,186 +62,218 @@ __device__ __forceinline__ int centred_mod(float x, float m, float inv_m, int lo
   if (r < lo) r += mi;
   return r;
 }
-// Recombine one element's accumulators (Eq. sq-shortcut / Eq. kar) plus the
-// previous slab's residue `prev`, and reduce.
-__device__ __forceinline__ int combine_residue(float a0, float a1, float a2, bool square, float s,
-                                               float m, float inv_m, int lo, int hi, int prev) {
-  float r0 = loose_mod(a0, m, inv_m);
-  float r1 = loose_mod(a1, m, inv_m);
-  float v;
-  if (square) {
-    v = fmaf(s, r1, r0);                          // d0e0 + s(d1e0 + d0e1), |v| < 2^16
-  } else {
-    float r2 = loose_mod(a2, m, inv_m);           // 2^b Σ + (1-2^b) d0e0 + (2^2b-2^b) d1e1, b = 4
-    v = fmaf(16.f, r0, fmaf(-15.f, r1, 240.f * r2));
-  }
+// Recombine one element's two accumulators (Eq. sq-shortcut, or Eq. kar with
+// the merged accumulator), add the previous slab's residue, and reduce.
+__device__ __forceinline__ int combine_residue(float a0, float a1, bool square, float s, float m, float inv_m,
+                                               int lo, int hi, int prev) {
+  const float r0 = loose_mod(a0, m, inv_m);
+  const float r1 = loose_mod(a1, m, inv_m);
+  // square: d0e0 + s(d1e0 + d0e1), |v| < 2^16
+  // nonsquare (b = 4): 2^b Σ + (1-2^b)(d0e0 - 2^b d1e1), |v| < 2^15
+  float v = square ? fmaf(s, r1, r0) : fmaf(16.f, r0, -15.f * r1);
   v += static_cast<float>(prev);
   return centred_mod(v, m, inv_m, lo, hi);
 }
 
 struct EpiCtx {
-  int16_t* res;        // r × (m×n, ld = m)
+  int16_t* res;   // r × (m×n, ld = m)
   float* urow;
   Oz2Device* dev;
   int64_t m, n;
 };
 
-// ---------------------------------------------------------------------------
+struct UnitMap {
+  int64_t ntm, ntn, ntiles, nunits;
+};
+
+// Unit u → modulus and tile (grouped raster of kGroupM tile rows).
+__device__ __forceinline__ void unit_coords(int64_t u, const UnitMap& um, int* modulus, int64_t* tm, int64_t* tn) {
+  *modulus = static_cast<int>(u / um.ntiles);
+  const int64_t t = u - static_cast<int64_t>(*modulus) * um.ntiles;
+  const int64_t per_group = kGroupM * um.ntn;
+  const int64_t g = t / per_group;
+  const int64_t first = g * kGroupM;
+  const int64_t gm = um.ntm - first < kGroupM ? um.ntm - first : kGroupM;
+  const int64_t local = t - g * per_group;
+  *tm = first + local % gm;
+  *tn = local / gm;
+}
+
 template <int MODE>
-__global__ void __launch_bounds__(kGemmThreads, 1)
-    plane_gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                         const __grid_constant__ Oz2Moduli mods, int64_t k_pad, EpiCtx ctx) {
-  using Cfg = GemmCfg<MODE>;
-  constexpr int S = Cfg::kStages, P = Cfg::kMaxP;
+__device__ __forceinline__ int planes_of(const Oz2Moduli& mods, int i) {
+  return MODE == 0 ? (mods.sq_base[i] ? 2 : 3) : 1;
+}
+template <int MODE>
+__device__ __forceinline__ int64_t slab_steps_of(const Oz2Moduli& mods, int i, int64_t ksteps) {
+  if (MODE == 1) return ksteps;
+  return (mods.sq_base[i] ? kKSlabSquare : kKSlabMerged) / kBK;
+}
+
+// MODE 0: residue planes (all moduli); MODE 1: magnitude planes ("+1" pass).
+template <int MODE>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
+    plane_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                      const __grid_constant__ Oz2Moduli mods, int64_t k_pad, UnitMap um, EpiCtx ctx) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* sA = smem;                                  // [S][P][16 KiB]
-  uint8_t* sB = smem + S * P * kTileBytes;             // [S][P][16 KiB]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sB + S * P * kTileBytes);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kStages * kStageBytes);
   // bars: full[S], empty[S], acc_full, acc_empty, drain
   __shared__ uint32_t tmem_base_s;
-  __shared__ int abort_s;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t m0 = static_cast<int64_t>(blockIdx.x) * kBM;
-  const int64_t n0 = static_cast<int64_t>(blockIdx.y) * kBN;
-  const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + S);
-  const uint32_t acc_full = smem_u32(bars + 2 * S), acc_empty = smem_u32(bars + 2 * S + 1);
-  const uint32_t drain_bar = smem_u32(bars + 2 * S + 2);
+  const uint32_t rank = cluster_ctarank();
+  const bool leader = rank == 0;
+  const int64_t pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
+  const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + kStages);
+  const uint32_t acc_full = smem_u32(bars + 2 * kStages), acc_empty = smem_u32(bars + 2 * kStages + 1);
+  const uint32_t drain_bar = smem_u32(bars + 2 * kStages + 2);
+  const int64_t ksteps = k_pad / kBK;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < S; ++s) {
+    for (int s = 0; s < kStages; ++s) {
       mbar_init(full0 + 8 * s, 1);
       mbar_init(empty0 + 8 * s, 1);
     }
     mbar_init(acc_full, 1);
-    mbar_init(acc_empty, 128);
+    mbar_init(acc_empty, 2 * kEpiWarps);
     mbar_init(drain_bar, 1);
-    abort_s = 0;
     fence_barrier_init();
-    fence_proxy_async_smem();
     prefetch_tensormap(&tmA);
     prefetch_tensormap(&tmB);
   }
   if (warp == 1) {
-    tmem_alloc(smem_u32(&tmem_base_s), Cfg::kTmemCols);
-    tmem_relinquish();
+    tmem_alloc_pair(smem_u32(&tmem_base_s), kTmemCols);
+    tmem_relinquish_pair();
   }
   tc_fence_before();
-  __syncthreads();
+  cluster_sync_all();
   tc_fence_after();
   const uint32_t tmem = tmem_base_s;
-
-  const int nmod = MODE == 0 ? mods.r : 1;
-  const int64_t ksteps = k_pad / kBK;
-  const int64_t slab_steps = MODE == 0 ? kKSlab / kBK : ksteps;
-  const int64_t nslabs = (ksteps + slab_steps - 1) / slab_steps;
+  bool ok = true;
 
   if (warp == 0) {
-    // ---------------- TMA producer ----------------
+    // ---------------- TMA producer (both CTAs) ----------------
     if (lane == 0) {
       uint32_t it = 0;
-      bool ok = true;
-      for (int i = 0; i < nmod && ok; ++i) {
-        const int np = MODE == 0 ? (mods.sq_base[i] ? 2 : 3) : 1;
+      const uint32_t full_leader0 = mapa_shared(full0, 0);
+      for (int64_t u = pair; u < um.nunits && ok; u += npairs) {
+        int i;
+        int64_t tm, tn;
+        unit_coords(u, um, &i, &tm, &tn);
+        const int np = planes_of<MODE>(mods, i);
         const int pbase = MODE == 0 ? mods.plane_off[i] : 0;
-        for (int64_t kb = 0; kb < ksteps && ok; ++kb, ++it) {
-          const int s = it % S;
-          const uint32_t ph = (it / S) & 1;
-          if (!mbar_wait_bounded(empty0 + 8 * s, ph ^ 1, kWaitLimit) || *reinterpret_cast<volatile int*>(&abort_s)) {
-            ok = false;
-            break;
-          }
-          mbar_arrive_expect_tx(full0 + 8 * s, 2u * np * kTileBytes);
-          for (int p = 0; p < np; ++p) {
-            tma_load_3d(smem_u32(sA + (s * P + p) * kTileBytes), &tmA, full0 + 8 * s,
-                        static_cast<int>(kb * kBK), static_cast<int>(m0), pbase + p);
-            tma_load_3d(smem_u32(sB + (s * P + p) * kTileBytes), &tmB, full0 + 8 * s,
-                        static_cast<int>(kb * kBK), static_cast<int>(n0), pbase + p);
+        const int ya = static_cast<int>(tm * kTileM + rank * kRows);
+        const int yb = static_cast<int>(tn * kTileN + rank * kRows);
+        for (int64_t kb = 0; kb < ksteps && ok; ++kb) {
+          for (int p = 0; p < np; ++p, ++it) {
+            const int s = it % kStages;
+            if (!mbar_wait_bounded(empty0 + 8 * s, ((it / kStages) & 1) ^ 1, kWaitLimit)) {
+              ok = false;
+              break;
+            }
+            if (leader) mbar_arrive_expect_tx(full0 + 8 * s, 2u * kStageBytes);
+            const uint32_t sa = smem_u32(smem + s * kStageBytes);
+            const int x = static_cast<int>(kb * kBK);
+            tma_load_3d_pair(sa, &tmA, full_leader0 + 8 * s, x, ya, pbase + p);
+            tma_load_3d_pair(sa + kTileBytes, &tmB, full_leader0 + 8 * s, x, yb, pbase + p);
           }
         }
       }
       if (!ok) {
-        atomicExch(&abort_s, 1);
         ctx.dev->status = kStatusTimeout;
         ctx.dev->timeout_site = 1;
       }
-      // Drain: wait (bounded) until every issued stage has landed.
-      for (uint32_t j = (it > S ? it - S : 0); j < it; ++j)
-        mbar_wait_bounded(full0 + 8 * (j % S), (j / S) & 1, kWaitLimit);
+      if (leader)  // the leader's stage barriers also count the peer's bytes
+        for (uint32_t j = (it > kStages ? it - kStages : 0); j < it; ++j)
+          mbar_wait_bounded(full0 + 8 * (j % kStages), (j / kStages) & 1, kWaitLimit);
     }
     __syncwarp();
   } else if (warp == 1) {
-    // ---------------- MMA issuer ----------------
-    if (lane == 0) {
-      constexpr uint32_t idesc = idesc_f8_f32(kBM, kBN);
+    // ---------------- MMA issuer (leader CTA) ----------------
+    if (leader && lane == 0) {
+      constexpr uint32_t idesc = idesc_f8_f32(kTileM, kTileN);
       uint32_t it = 0, accph = 0;
-      bool ok = true;
-      for (int i = 0; i < nmod && ok; ++i) {
-        const bool square = MODE == 0 ? mods.sq_base[i] != 0 : true;
-        const int np = MODE == 0 ? (square ? 2 : 3) : 1;
-        for (int64_t sl = 0; sl < nslabs && ok; ++sl) {
-          if (!mbar_wait_bounded(acc_empty, accph ^ 1, kWaitLimit) || *reinterpret_cast<volatile int*>(&abort_s)) {
+      auto wait_full = [&](uint32_t j) {
+        return mbar_wait_bounded(full0 + 8 * (j % kStages), (j / kStages) & 1, kWaitLimit);
+      };
+      auto desc = [&](uint32_t j, int operand, int kk) {
+        return smem_desc_sw128(smem_u32(smem + (j % kStages) * kStageBytes + operand * kTileBytes) + kk * 32);
+      };
+      for (int64_t u = pair; u < um.nunits && ok; u += npairs) {
+        int i;
+        int64_t tm, tn;
+        unit_coords(u, um, &i, &tm, &tn);
+        const int np = planes_of<MODE>(mods, i);
+        const int64_t slab = slab_steps_of<MODE>(mods, i, ksteps);
+        for (int64_t kb0 = 0; kb0 < ksteps && ok; kb0 += slab) {
+          if (!mbar_wait_bounded(acc_empty, accph ^ 1, kWaitLimit)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const int64_t kb0 = sl * slab_steps, kb1 = min(ksteps, kb0 + slab_steps);
-          for (int64_t kb = kb0; kb < kb1; ++kb, ++it) {
-            const int s = it % S;
-            const uint32_t ph = (it / S) & 1;
-            if (!mbar_wait_bounded(full0 + 8 * s, ph, kWaitLimit) || *reinterpret_cast<volatile int*>(&abort_s)) {
-              ok = false;
-              break;
-            }
-            tc_fence_after();
-            const uint32_t a0 = smem_u32(sA + (s * P) * kTileBytes);
-            const uint32_t b0 = smem_u32(sB + (s * P) * kTileBytes);
+          const int64_t kb1 = min(ksteps, kb0 + slab);
+          for (int64_t kb = kb0; kb < kb1 && ok; ++kb) {
+            const uint32_t first = kb == kb0 ? 0u : 1u;
+            if (np == 2) {  // square: stages (d0,e0) and (d1,e1)
+              if (!wait_full(it) || !wait_full(it + 1)) {
+                ok = false;
+                break;
+              }
+              tc_fence_after();
 #pragma unroll
-            for (int kk = 0; kk < kBK / 32; ++kk) {
-              const uint32_t first = (kb == kb0 && kk == 0) ? 0u : 1u;
-              const uint32_t off = kk * 32;
-              auto da = [&](int p) { return smem_desc_sw128(a0 + p * kTileBytes + off); };
-              auto db = [&](int p) { return smem_desc_sw128(b0 + p * kTileBytes + off); };
-              if (MODE == 1) {
-                mma_f8(tmem, da(0), db(0), idesc, first);
-              } else if (np == 2) {
-                mma_f8(tmem + 0 * kBN, da(0), db(0), idesc, first);  // d0·e0
-                mma_f8(tmem + 1 * kBN, da(1), db(0), idesc, first);  // d1·e0
-                mma_f8(tmem + 1 * kBN, da(0), db(1), idesc, 1u);     // + d0·e1
-              } else {
-                mma_f8(tmem + 0 * kBN, da(0), db(0), idesc, first);  // (d0+d1)(e0+e1)
-                mma_f8(tmem + 1 * kBN, da(1), db(1), idesc, first);  // d0·e0
-                mma_f8(tmem + 2 * kBN, da(2), db(2), idesc, first);  // d1·e1
+              for (int kk = 0; kk < kBK / 32; ++kk) {
+                const uint32_t acc = kk ? 1u : first;
+                mma_f8_pair(tmem, desc(it, 0, kk), desc(it, 1, kk), idesc, acc);                   // d0·e0
+                mma_f8_pair(tmem + kAccCols, desc(it + 1, 0, kk), desc(it, 1, kk), idesc, acc);    // d1·e0
+                mma_f8_pair(tmem + kAccCols, desc(it, 0, kk), desc(it + 1, 1, kk), idesc, 1u);     // + d0·e1
+              }
+              mma_commit_pair_mc(empty0 + 8 * (it % kStages), 0x3);
+              mma_commit_pair_mc(empty0 + 8 * ((it + 1) % kStages), 0x3);
+              it += 2;
+            } else {
+              for (int p = 0; p < np; ++p, ++it) {  // nonsquare: Σ·Σ → acc0; d0e0, -16 d1·e1 → acc1
+                if (!wait_full(it)) {
+                  ok = false;
+                  break;
+                }
+                tc_fence_after();
+                const uint32_t col = p == 0 ? 0u : kAccCols;
+#pragma unroll
+                for (int kk = 0; kk < kBK / 32; ++kk) {
+                  const uint32_t acc = (kk || p == 2) ? 1u : first;
+                  mma_f8_pair(tmem + col, desc(it, 0, kk), desc(it, 1, kk), idesc, acc);
+                }
+                mma_commit_pair_mc(empty0 + 8 * (it % kStages), 0x3);
               }
             }
-            mma_commit(empty0 + 8 * s);     // stage free once these MMAs retire
           }
           if (!ok) break;
-          mma_commit(acc_full);             // accumulators complete for this slab
+          mma_commit_pair_mc(acc_full, 0x3);  // accumulators complete for this slab, both CTAs
           accph ^= 1;
         }
       }
       if (!ok) {
-        atomicExch(&abort_s, 1);
         ctx.dev->status = kStatusTimeout;
         ctx.dev->timeout_site = 2;
       }
-      // Drain outstanding MMAs before the TMEM is released, through a barrier
-      // of its own: an extra arrival on acc_full could complete a phase
-      // beyond the one the epilogue is polling and alias its parity.
-      mma_commit(drain_bar);
+      // All MMAs retired before the tensor memory or the peer's shared memory goes away.
+      mma_commit_pair(drain_bar);
       mbar_wait_bounded(drain_bar, 0, kWaitLimit);
     }
     __syncwarp();
   } else {
-    // ---------------- epilogue (warps 2..5) ----------------
-    const int q = warp & 3;                         // TMEM lane quarter
-    const int64_t row = m0 + 32 * q + lane;
-    const uint32_t lane_addr = tmem + (static_cast<uint32_t>(32 * q) << 16);
+    // ---------------- epilogue (warps 2..9, both CTAs) ----------------
+    const int q = warp & 3;                    // TMEM lane quarter of this warp
+    const int h = (warp - 2) >> 2;             // column half
+    const uint32_t lane_addr = tmem + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(128 * h);
+    const uint32_t acc_empty_leader = mapa_shared(acc_empty, 0);
     uint32_t accph = 0;
-    bool ok = true;
-    for (int i = 0; i < nmod && ok; ++i) {
+    for (int64_t u = pair; u < um.nunits && ok; u += npairs) {
+      int i;
+      int64_t tm, tn;
+      unit_coords(u, um, &i, &tm, &tn);
+      const int64_t row = tm * kTileM + rank * kRows + 32 * q + lane;
+      const int64_t col0 = tn * kTileN + 128 * h;
       const bool square = MODE == 0 ? mods.sq_base[i] != 0 : true;
       const float mf = MODE == 0 ? static_cast<float>(mods.m[i]) : 1.f;
       const float inv = 1.f / mf;
@@ -245,20 +281,18 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       const int lo = MODE == 0 ? -(mods.m[i] / 2) : 0;
       const int hi = MODE == 0 ? mods.m[i] - 1 - mods.m[i] / 2 : 0;
       int16_t* resi = MODE == 0 ? ctx.res + static_cast<size_t>(i) * ctx.m * ctx.n : nullptr;
-      for (int64_t sl = 0; sl < nslabs; ++sl) {
-        if (!mbar_wait_bounded(acc_full, accph, kWaitLimit) || *reinterpret_cast<volatile int*>(&abort_s)) {
+      const int64_t slab = slab_steps_of<MODE>(mods, i, ksteps);
+      float rowmax = 0.f;
+      for (int64_t kb0 = 0; kb0 < ksteps; kb0 += slab) {
+        if (!mbar_wait_bounded(acc_full, accph, kWaitLimit)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        float rowmax = 0.f;
-        for (int c = 0; c < kBN; c += 32) {
-          uint32_t v0[32], v1[32], v2[32];
+        for (int c = 0; c < 128; c += 32) {
+          uint32_t v0[32], v1[32];
           tmem_ld32(lane_addr + c, v0);
-          if (MODE == 0) {
-            tmem_ld32(lane_addr + kBN + c, v1);
-            if (!square) tmem_ld32(lane_addr + 2 * kBN + c, v2);
-          }
+          if (MODE == 0) tmem_ld32(lane_addr + kAccCols + c, v1);
           tmem_ld_wait();
           if (MODE == 1) {
 #pragma unroll
@@ -266,38 +300,37 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           } else if (row < ctx.m) {
 #pragma unroll
             for (int j = 0; j < 32; ++j) {
-              const int64_t col = n0 + c + j;
+              const int64_t col = col0 + c + j;
               if (col < ctx.n) {
                 int16_t* dst = resi + col * ctx.m + row;
-                const int prev = sl ? *dst : 0;
-                const float a2 = square ? 0.f : __uint_as_float(v2[j]);
-                *dst = static_cast<int16_t>(combine_residue(__uint_as_float(v0[j]), __uint_as_float(v1[j]),
-                                                            a2, square, sb, mf, inv, lo, hi, prev));
+                const int prev = kb0 ? *dst : 0;
+                *dst = static_cast<int16_t>(combine_residue(__uint_as_float(v0[j]), __uint_as_float(v1[j]), square,
+                                                            sb, mf, inv, lo, hi, prev));
               }
             }
           }
         }
-        if (MODE == 1) {
-          // rows past m hold zeros (TMA fills out-of-range rows with 0)
-          if (row < ctx.m) atomicMax(reinterpret_cast<int*>(ctx.urow) + row, __float_as_int(rowmax));
-          const int wm = __reduce_max_sync(0xffffffffu, __float_as_int(rowmax));
-          if (lane == 0) atomicMax(&ctx.dev->u_max_bits, wm);
-        }
         tc_fence_before();
-        mbar_arrive(acc_empty);
+        __syncwarp();
+        if (lane == 0) mbar_arrive_remote(acc_empty_leader);
         accph ^= 1;
+      }
+      if (MODE == 1 && ok) {
+        // rows past m hold zeros (TMA fills out-of-range rows with 0)
+        if (row < ctx.m) atomicMax(reinterpret_cast<int*>(ctx.urow) + row, __float_as_int(rowmax));
+        const int wm = __reduce_max_sync(0xffffffffu, __float_as_int(rowmax));
+        if (lane == 0) atomicMax(&ctx.dev->u_max_bits, wm);
       }
     }
     if (!ok) {
-      atomicExch(&abort_s, 1);
       ctx.dev->status = kStatusTimeout;
       ctx.dev->timeout_site = 3;
     }
   }
   tc_fence_before();
-  __syncthreads();
+  cluster_sync_all();  // neither CTA leaves while the pair's MMAs or loads may touch it
   tc_fence_after();
-  if (warp == 1) tmem_dealloc(tmem, Cfg::kTmemCols);
+  if (warp == 1) tmem_dealloc_pair(tmem, kTmemCols);
 }
 
 // ---------------------------------------------------------------------------
@@ -313,8 +346,7 @@ __device__ __forceinline__ float e4m3_to_float(uint8_t c) {
 
 template <int MODE>
 __global__ void plane_gemm_simt_kernel(const uint8_t* __restrict__ pa, const uint8_t* __restrict__ pb,
-                                       const __grid_constant__ Oz2Moduli mods, int64_t k_pad,
-                                       EpiCtx ctx) {
+                                       const __grid_constant__ Oz2Moduli mods, int64_t k_pad, EpiCtx ctx) {
   const int64_t row = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   const int64_t col = blockIdx.y;
   if (row >= ctx.m || col >= ctx.n) return;
@@ -334,10 +366,11 @@ __global__ void plane_gemm_simt_kernel(const uint8_t* __restrict__ pa, const uin
     const float inv = 1.f / mf;
     const int lo = -(mods.m[i] / 2), hi = mods.m[i] - 1 - mods.m[i] / 2;
     const size_t p0 = mods.plane_off[i];
+    const int64_t slab = square ? kKSlabSquare : kKSlabMerged;
     int res = 0;
-    for (int64_t l0 = 0; l0 < k_pad; l0 += kKSlab) {
-      float a0 = 0.f, a1 = 0.f, a2 = 0.f;
-      const int64_t l1 = min(k_pad, l0 + kKSlab);
+    for (int64_t l0 = 0; l0 < k_pad; l0 += slab) {
+      float a0 = 0.f, a1 = 0.f;
+      const int64_t l1 = min(k_pad, l0 + slab);
       for (int64_t l = l0; l < l1; ++l) {
         const float x0 = e4m3_to_float(ar[p0 * sa + l]), y0 = e4m3_to_float(bc[p0 * sbs + l]);
         const float x1 = e4m3_to_float(ar[(p0 + 1) * sa + l]), y1 = e4m3_to_float(bc[(p0 + 1) * sbs + l]);
@@ -347,11 +380,10 @@ __global__ void plane_gemm_simt_kernel(const uint8_t* __restrict__ pa, const uin
         } else {
           const float x2 = e4m3_to_float(ar[(p0 + 2) * sa + l]), y2 = e4m3_to_float(bc[(p0 + 2) * sbs + l]);
           a0 += x0 * y0;
-          a1 += x1 * y1;
-          a2 += x2 * y2;
+          a1 += x1 * y1 + x2 * y2;
         }
       }
-      res = combine_residue(a0, a1, a2, square, static_cast<float>(mods.sq_base[i]), mf, inv, lo, hi, res);
+      res = combine_residue(a0, a1, square, static_cast<float>(mods.sq_base[i]), mf, inv, lo, hi, res);
     }
     ctx.res[static_cast<size_t>(i) * ctx.m * ctx.n + col * ctx.m + row] = static_cast<int16_t>(res);
   }
@@ -377,14 +409,15 @@ static EncodeTiledFn get_encode_fn() {
   return fn;
 }
 
-// Planes of one operand: `np` planes of rows × k_pad bytes, row-major.
+// Planes of one operand: `np` planes of rows × k_pad bytes, row-major; the
+// box is 128 rows × 128 bytes with the 128-byte swizzle the MMA descriptors use.
 static bool make_plane_map(CUtensorMap* map, const uint8_t* base, int64_t rows, int64_t k_pad, int np) {
   EncodeTiledFn enc = get_encode_fn();
   if (!enc) return false;
   cuuint64_t dims[3] = {static_cast<cuuint64_t>(k_pad), static_cast<cuuint64_t>(rows),
                         static_cast<cuuint64_t>(np)};
   cuuint64_t strides[2] = {static_cast<cuuint64_t>(k_pad), static_cast<cuuint64_t>(rows * k_pad)};
-  cuuint32_t box[3] = {kBK, static_cast<cuuint32_t>(kBM), 1};
+  cuuint32_t box[3] = {kBK, static_cast<cuuint32_t>(kRows), 1};
   cuuint32_t estr[3] = {1, 1, 1};
   CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, const_cast<uint8_t*>(base), dims, strides, box, estr,
                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -392,10 +425,13 @@ static bool make_plane_map(CUtensorMap* map, const uint8_t* base, int64_t rows, 
   return r == CUDA_SUCCESS;
 }
 
-template <int MODE>
-static size_t gemm_smem_bytes() {
-  using Cfg = GemmCfg<MODE>;
-  return 1024 + 2 * static_cast<size_t>(Cfg::kStages) * Cfg::kMaxP * kTileBytes + 8 * (2 * Cfg::kStages + 3);
+static size_t gemm_smem_bytes() { return 1024 + static_cast<size_t>(kStages) * kStageBytes + 8 * (2 * kStages + 3); }
+
+static int num_sms() {
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  return sms;
 }
 
 // mode: 0 residues (tensor cores), 1 magnitude (tensor cores),
@@ -416,23 +452,38 @@ cudaError_t launch_plane_gemm(int64_t m, int64_t n, int64_t k_pad, const Oz2Modu
   CUtensorMap ta, tb;
   if (!make_plane_map(&ta, planes_a, m, k_pad, np) || !make_plane_map(&tb, planes_b, n, k_pad, np))
     return cudaErrorInvalidValue;
-  dim3 g(static_cast<unsigned>((m + kBM - 1) / kBM), static_cast<unsigned>((n + kBN - 1) / kBN));
-  cudaError_t err;
-  if (mode == 0) {
-    size_t smem = gemm_smem_bytes<0>();
-    if ((err = cudaFuncSetAttribute(plane_gemm_tc_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    static_cast<int>(smem))) != cudaSuccess)
-      return err;
-    count_launch();
-    plane_gemm_tc_kernel<0><<<g, kGemmThreads, smem, st>>>(ta, tb, mods, k_pad, ctx);
-  } else {
-    size_t smem = gemm_smem_bytes<1>();
-    if ((err = cudaFuncSetAttribute(plane_gemm_tc_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    static_cast<int>(smem))) != cudaSuccess)
-      return err;
-    count_launch();
-    plane_gemm_tc_kernel<1><<<g, kGemmThreads, smem, st>>>(ta, tb, mods, k_pad, ctx);
+  UnitMap um;
+  um.ntm = (m + kTileM - 1) / kTileM;
+  um.ntn = (n + kTileN - 1) / kTileN;
+  um.ntiles = um.ntm * um.ntn;
+  um.nunits = um.ntiles * (mode == 0 ? mods.r : 1);
+  const size_t smem = gemm_smem_bytes();
+  auto kern = mode == 0 ? plane_gemm_kernel<0> : plane_gemm_kernel<1>;
+  cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  if (err != cudaSuccess) return err;
+  // Persistent grid: as many CTA pairs as can be resident at once.
+  int64_t pairs = num_sms() / 2;
+  {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(2 * pairs));
+    cfg.blockDim = dim3(kGemmThreads);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeClusterDimension;
+    attr.val.clusterDim.x = 2;
+    attr.val.clusterDim.y = 1;
+    attr.val.clusterDim.z = 1;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    int clusters = 0;
+    if (cudaOccupancyMaxActiveClusters(&clusters, kern, &cfg) == cudaSuccess && clusters > 0)
+      pairs = std::min<int64_t>(pairs, clusters);
+    else
+      cudaGetLastError();
   }
+  pairs = std::max<int64_t>(1, std::min<int64_t>(pairs, um.nunits));
+  count_launch();
+  kern<<<static_cast<unsigned>(2 * pairs), kGemmThreads, smem, st>>>(ta, tb, mods, k_pad, um, ctx);
   return cudaGetLastError();
 }
 

@@ -18,8 +18,9 @@ static const int kModuliAll[kMaxModuli] = {1089, 1024, 961, 841, 625, 529, 511, 
                                            503,  499,  491, 487, 479, 467, 463, 461};
 constexpr int kTableMax = 10240;  // Σ of all sixteen moduli = 9939 entries
 
-// Packed E4M3 digit planes of every residue (byte p = plane p), per modulus.
-static __device__ uint32_t g_plane_table[kTableMax];
+// Packed E4M3 digit planes of every residue (byte p = plane p), per modulus;
+// table 0 for A (last nonsquare plane pre-scaled by -16), table 1 for B.
+static __device__ uint32_t g_plane_table[2][kTableMax];
 // Device status block (sticky status word, fallback counts, scale summary).
 static __device__ Oz2Device g_status;
 
@@ -55,8 +56,11 @@ static int floor_mod(int a, int m) {
   return r < 0 ? r + m : r;
 }
 
-// Digit planes of the centred residue d (§2.5).
-static uint32_t plane_word(int d, int m) {
+// Digit planes of the centred residue d (§2.5).  With `merged` (the A
+// operand) the last nonsquare plane is stored as -16·d1, the accumulator
+// merge of §2.5: the products d0·e0 and (-16 d1)·e1 then share the weight
+// (1 - 2^b) in one accumulator.
+static uint32_t plane_word(int d, int m, bool merged) {
   int s = isqrt_exact(m);
   int p[3] = {0, 0, 0}, np;
   if (s) {  // balanced base s: d0 ∈ [-⌊s/2⌋, s-1-⌊s/2⌋]
@@ -76,7 +80,7 @@ static uint32_t plane_word(int d, int m) {
     }
     p[0] = d0 + d1;
     p[1] = d0;
-    p[2] = d1;
+    p[2] = merged ? -16 * d1 : d1;
     np = 3;
   }
   uint32_t w = 0;
@@ -168,7 +172,8 @@ static Oz2Moduli build_moduli(int r, int quant) {
 // ---------------------------------------------------------------------------
 struct DeviceState {
   bool ready = false;
-  uint32_t* table = nullptr;
+  uint32_t* table_a = nullptr;
+  uint32_t* table_b = nullptr;
   Oz2Device* status = nullptr;
 };
 static DeviceState g_devs[64];
@@ -212,26 +217,30 @@ static int device_state(DeviceState** out) {
   std::lock_guard<std::mutex> lk(g_mu);
   DeviceState& s = g_devs[dev];
   if (!s.ready) {
-    static uint32_t host_table[kTableMax];
-    int off = 0;
-    for (int i = 0; i < kMaxModuli; ++i) {
-      const int m = kModuliAll[i];
-      for (int r = 0; r < m; ++r) {
-        int d = r > m - 1 - m / 2 ? r - m : r;  // centred residue
-        uint32_t w = plane_word(d, m);
-        if (w == 0xFFFFFFFFu) return OZ2_ERR_CUDA;
-        host_table[off + r] = w;
+    static uint32_t host_table[2][kTableMax];
+    for (int t = 0; t < 2; ++t) {
+      int off = 0;
+      for (int i = 0; i < kMaxModuli; ++i) {
+        const int m = kModuliAll[i];
+        for (int r = 0; r < m; ++r) {
+          int d = r > m - 1 - m / 2 ? r - m : r;  // centred residue
+          uint32_t w = plane_word(d, m, t == 0);
+          if (w == 0xFFFFFFFFu) return OZ2_ERR_CUDA;
+          host_table[t][off + r] = w;
+        }
+        off += m;
       }
-      off += m;
     }
-    if (cudaMemcpyToSymbol(g_plane_table, host_table, sizeof(uint32_t) * off) != cudaSuccess)
-      return OZ2_ERR_CUDA;
+    if (cudaMemcpyToSymbol(g_plane_table, host_table, sizeof(host_table)) != cudaSuccess) return OZ2_ERR_CUDA;
     Oz2Device zero;
     std::memset(&zero, 0, sizeof(zero));
     if (cudaMemcpyToSymbol(g_status, &zero, sizeof(zero)) != cudaSuccess) return OZ2_ERR_CUDA;
-    if (cudaGetSymbolAddress(reinterpret_cast<void**>(&s.table), g_plane_table) != cudaSuccess ||
+    uint32_t* tables = nullptr;
+    if (cudaGetSymbolAddress(reinterpret_cast<void**>(&tables), g_plane_table) != cudaSuccess ||
         cudaGetSymbolAddress(reinterpret_cast<void**>(&s.status), g_status) != cudaSuccess)
       return OZ2_ERR_CUDA;
+    s.table_a = tables;
+    s.table_b = tables + kTableMax;
     s.ready = true;
   }
   *out = &s;
@@ -408,7 +417,7 @@ int oz2_dgemm_ex(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, 
   if (err == cudaSuccess) err = launch_choose_scales(m, n, k, mods, scale, urow, ra, cb, rf, cf, d, e, ds->status, s);
   mark(4);
   if (err == cudaSuccess)
-    err = launch_deconstruct(m, n, k, mods, ds->table, A, lda, B, ldb, d, e, rf, cf, quant, pa, pb, s);
+    err = launch_deconstruct(m, n, k, mods, ds->table_a, ds->table_b, A, lda, B, ldb, d, e, rf, cf, quant, pa, pb, s);
   mark(5);
   if (err == cudaSuccess)
     err = launch_plane_gemm(m, n, L.k_pad, mods, pa, pb, simt ? 2 : 0, res, nullptr, ds->status, s);
@@ -418,7 +427,7 @@ int oz2_dgemm_ex(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, 
   if (err == cudaSuccess) err = launch_fallback_lists(m, n, k, A, lda, B, ldb, rf, cf, misc, C, ldc, s);
   mark(8);
 
-  hs.k_slab = static_cast<int>(std::min<int64_t>(kKSlab, L.k_pad));
+  hs.k_slab = static_cast<int>(std::min<int64_t>(kKSlabMerged, L.k_pad));
   if (ts) ts->pending = true;
   return to_status(err);
 }
@@ -589,7 +598,7 @@ int oz2_deconstruct(int64_t m, int64_t n, int64_t k, int num_moduli, const doubl
   DeviceState* ds = nullptr;
   if ((st = device_state(&ds)) != OZ2_OK) return st;
   const Oz2Moduli mods = build_moduli(num_moduli, quant);
-  return to_status(launch_deconstruct(m, n, k, mods, ds->table, A, lda, B, ldb, d, e, row_flag, col_flag, quant,
+  return to_status(launch_deconstruct(m, n, k, mods, ds->table_a, ds->table_b, A, lda, B, ldb, d, e, row_flag, col_flag, quant,
                                       planes_a, planes_b, static_cast<cudaStream_t>(stream)));
 }
 

@@ -18,10 +18,12 @@ constexpr int kMaxPlanes = 48;         // 3 per modulus at most
 constexpr int kKPad = 128;             // k is padded to a multiple of this
 constexpr int kMagClampMax = 9;        // 2^-9: smallest E4M3 magnitude
 constexpr int kFallbackWindow = 128;   // binades from the median (fallback)
-// Exact FP32 accumulation (Eq. accum-exact): every accumulator term is at
-// most 512 in magnitude (square cross term d1e0 + d0e1; nonsquare terms are
-// ≤ 484), so K_slab · 512 ≤ 2^24 holds for K_slab = 32768.
-constexpr int kKSlab = 32768;
+// Exact FP32 accumulation (Eq. accum-exact), K_slab · max|term| ≤ 2^24:
+//  square moduli: terms d0e0 (≤ 256) and d1e0 + d0e1 (≤ 512) → K_slab 32768;
+//  nonsquare moduli with the merged accumulator d0e0 - 16·d1e1 (≤ 4095 on
+//  the S tail and the extension primes) → K_slab 4096 (4096 · 4095 < 2^24).
+constexpr int kKSlabSquare = 32768;
+constexpr int kKSlabMerged = 4096;
 
 // Device status word values (stored in Oz2Device::status).
 constexpr int kStatusTimeout = 1;
@@ -134,6 +136,71 @@ __device__ __forceinline__ void prefetch_tensormap(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
 }
 
+// --- clusters (CTA pairs) ----------------------------------------------------
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// shared::cluster address of the same shared-memory offset in CTA `rank`.
+__device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// Arrive on an mbarrier of another CTA of the cluster (address from mapa_shared).
+__device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+// 3-D tiled TMA load issued by either CTA of a pair; the transaction bytes
+// complete on `bar` (a shared::cluster address, here the leader CTA's barrier).
+__device__ __forceinline__ void tma_load_3d_pair(uint32_t dst, const CUtensorMap* map, uint32_t bar, int x, int y,
+                                                 int z) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cta.global.tile.mbarrier::complete_tx::bytes.cta_group::2"
+      " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(x), "r"(y), "r"(z)
+      : "memory");
+}
+
+// --- tcgen05, CTA pair (cta_group::2) -------------------------------------------
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish_pair() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+// D[tmem] (+)= A·Bᵀ over the CTA pair (M = 256: 128 rows of A in each CTA's
+// shared memory at the same offset; B split likewise), issued by the leader.
+__device__ __forceinline__ void mma_f8_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                            uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::2.kind::f8f6f4 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// Arrive once on the barrier at this shared offset in every CTA of `mask`
+// when all prior tcgen05 ops of the issuing thread complete.
+__device__ __forceinline__ void mma_commit_pair_mc(uint32_t bar, uint16_t mask) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+          bar),
+      "h"(mask)
+      : "memory");
+}
+__device__ __forceinline__ void mma_commit_pair(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+               : "memory");
+}
+
 // --- tcgen05 -----------------------------------------------------------------
 __device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem),
@@ -236,7 +303,8 @@ cudaError_t launch_choose_scales(int64_t m, int64_t n, int64_t k, const Oz2Modul
                                  const uint8_t* col_flag, int32_t* d, int32_t* e,
                                  Oz2Device* dev, cudaStream_t st);
 cudaError_t launch_deconstruct(int64_t m, int64_t n, int64_t k, const Oz2Moduli& mods,
-                               const uint32_t* table, const double* A, int64_t lda,
+                               const uint32_t* table_a, const uint32_t* table_b,
+                               const double* A, int64_t lda,
                                const double* B, int64_t ldb, const int32_t* d, const int32_t* e,
                                const uint8_t* row_flag, const uint8_t* col_flag, int quant,
                                uint8_t* planes_a, uint8_t* planes_b, cudaStream_t st);

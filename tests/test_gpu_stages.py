@@ -99,7 +99,7 @@ def test_deconstruct(oz, shape, r, quant):
     pa, pb = oz.oz2_deconstruct(dA, dB, d, e, rf, cf, num_moduli=r, quant=quant)
     k_pad = (k + 127) // 128 * 128
     mods = orc.moduli(r)
-    want_a = planes_from_residues([orc.centred(res.At, mi) for mi in mods], mods, orc, k_pad)
+    want_a = planes_from_residues([orc.centred(res.At, mi) for mi in mods], mods, orc, k_pad, merged=True)
     want_b = planes_from_residues([orc.centred(res.Bt.T, mi) for mi in mods], mods, orc, k_pad)
     assert np.array_equal(pa.cpu().numpy(), want_a)
     assert np.array_equal(pb.cpu().numpy(), want_b)
@@ -110,7 +110,7 @@ def _residue_case(oz, m, n, k, r, gen, simt=False):
     k_pad = (k + 127) // 128 * 128
     a = [gen(mi, (m, k), 0) for mi in mods]
     b = [gen(mi, (n, k), 1) for mi in mods]
-    pa = planes_from_residues(a, mods, orc, k_pad)
+    pa = planes_from_residues(a, mods, orc, k_pad, merged=True)   # A: last nonsquare plane is -16·d1
     pb = planes_from_residues(b, mods, orc, k_pad)
     import torch
     got = oz.oz2_residue_gemm(torch.from_numpy(pa).cuda(), torch.from_numpy(pb).cuda(), m, n, k, r, simt=simt)
@@ -133,9 +133,38 @@ def test_residue_gemm_uniform(oz, shape, r, simt):
     _residue_case(oz, *shape, r, _uniform(sum(shape) + r), simt=simt)
 
 
-def test_residue_gemm_two_k_slabs(oz):
-    """k above the 32768-entry K-slab: the epilogue folds the slabs mod m."""
+def test_residue_gemm_k_slabs(oz):
+    """k above the K-slabs (32768 for squares, 4096 for nonsquare moduli): the
+    epilogue folds the slabs mod m."""
     _residue_case(oz, 128, 136, 33000, 4, _uniform(5))
+    _residue_case(oz, 300, 260, 9000, 8, _uniform(6))
+
+
+def _merged_argmax(m):
+    """Centred residues (d, e) maximising |d0e0 - 16 d1e1| for a nonsquare m."""
+    d = np.arange(-(m // 2), m - m // 2)
+    d0, d1 = orc.nonsquare_digits(d)
+    t = np.abs(d0[:, None] * d0[None, :] - 16 * d1[:, None] * d1[None, :])
+    i, j = np.unravel_index(np.argmax(t), t.shape)
+    return int(d[i]), int(d[j]), int(t[i, j])
+
+
+def test_residue_gemm_merged_accumulator_worst_case(oz):
+    """The merged nonsquare accumulator at its bound: 4096 terms of 4095
+    (Eq. accum-exact with K_slab = 4096), then a second slab."""
+    mods = orc.moduli(12)
+
+    def gen(mi, shape, side):
+        rows, kk = shape
+        if orc.square_base(mi):
+            return np.full(shape, mi // 2, dtype=np.int64)
+        d, e, t = _merged_argmax(mi)
+        assert t >= 3900
+        out = np.full(shape, d if side == 0 else e, dtype=np.int64)
+        out[1::2, 4096:] = -out[1::2, 4096:]
+        return out
+
+    _residue_case(oz, 256, 256, 8192, 12, gen)
 
 
 def test_residue_gemm_accumulator_extremes(oz):
