@@ -260,8 +260,8 @@ def oz2_deconstruct(A, B, d, e, rf, cf, num_moduli=12, quant="tz", stream=None):
 
 
 def oz2_residue_gemm(planes_a, planes_b, m, n, k, num_moduli=12, simt=False, stream=None):
-    """planes: uint8 CUDA tensors (P, rows, k_pad). Returns int16 (r, n, m) = r column-major m×n."""
-    res = torch.empty((num_moduli, n, m), dtype=torch.int16, device=planes_a.device)
+    """planes: uint8 CUDA tensors (P, rows, k_pad). Returns int16 (r, m, n): r row-major m×n."""
+    res = torch.empty((num_moduli, m, n), dtype=torch.int16, device=planes_a.device)
     fn = lib().oz2_residue_gemm_simt if simt else lib().oz2_residue_gemm
     _check(fn(m, n, k, num_moduli, _ptr(planes_a), _ptr(planes_b), _ptr(res), _stream(stream)),
            "oz2_residue_gemm")
@@ -269,10 +269,10 @@ def oz2_residue_gemm(planes_a, planes_b, m, n, k, num_moduli=12, simt=False, str
 
 
 def oz2_reconstruct(residues, d, e, m, n, num_moduli=12, C=None, stream=None):
-    """residues: int16 CUDA tensor (r, n, m) (column-major m×n per modulus)."""
+    """residues: int16 CUDA tensor (r, m, n) (row-major m×n per modulus)."""
     if C is None:
         C = torch.empty((n, m), dtype=torch.float64, device=residues.device).t()
-    _check(lib().oz2_reconstruct(m, n, num_moduli, _ptr(residues), m, _ptr(d), _ptr(e), _ptr(C), _ld(C),
+    _check(lib().oz2_reconstruct(m, n, num_moduli, _ptr(residues), n, _ptr(d), _ptr(e), _ptr(C), _ld(C),
                                  _stream(stream)), "oz2_reconstruct")
     return C
 
@@ -313,5 +313,5 @@ def workspace_views(ws: torch.Tensor, m: int, n: int, k: int, num_moduli: int) -
         "mag_b": view(L["mag_b"], n * k_pad, torch.uint8, (n, k_pad)),
         "planes_a": view(L["planes_a"], P * m * k_pad, torch.uint8, (P, m, k_pad)),
         "planes_b": view(L["planes_b"], P * n * k_pad, torch.uint8, (P, n, k_pad)),
-        "residues": view(L["residues"], num_moduli * m * n, torch.int16, (num_moduli, n, m)),
+        "residues": view(L["residues"], num_moduli * m * n, torch.int16, (num_moduli, m, n)),
     }

@@ -3,231 +3,233 @@
 // X = Σ v_k P_{k-1} mapped to [-M/2, M/2), and one correctly rounded
 // (round-to-nearest-even) conversion of X·2^-(d_i+e_j) to FP64, including
 // the subnormal range.
+//
+// Residues arrive row-major (r matrices of m×n, ld = ldr ≥ n) from the
+// residue GEMM; C is column-major.  A block computes a 32-row × 128-column
+// tile: each thread reads four consecutive residues of one row per modulus
+// (8-byte loads along n), computes its outputs, and the tile is transposed
+// through shared memory so that C is written in 256-byte column segments.
 #include "oz2_common.cuh"
 
 namespace oz2 {
 
 typedef unsigned long long u64;
-typedef unsigned int u32;
+typedef unsigned __int128 u128;
 
-// X (3 limbs, little-endian) = X·m + v.
-__device__ __forceinline__ void mul_add(u64 (&x)[3], uint32_t m, uint32_t v, bool three) {
-  u64 lo = x[0] * m;
-  u64 c = __umul64hi(x[0], m);
-  u64 s0 = lo + v;
-  c += s0 < lo;
-  u64 l1 = x[1] * m;
-  u64 c1 = __umul64hi(x[1], m);
-  u64 s1 = l1 + c;
-  c1 += s1 < l1;
-  x[0] = s0;
-  x[1] = s1;
-  if (three) x[2] = x[2] * m + c1;
+constexpr int kCrtRows = 32, kCrtCols = 128, kCrtThreads = 256;
+
+// X (L little-endian 32-bit limbs) = X·m + v.  Only the low `nl` limbs can be
+// nonzero afterwards; each limb step is one 32×32+64-bit multiply-add.
+template <int L>
+__device__ __forceinline__ void horner_step(uint32_t (&w)[L], int nl, uint32_t m, uint32_t v) {
+  u64 t = static_cast<u64>(w[0]) * m + v;
+  w[0] = static_cast<uint32_t>(t);
+#pragma unroll
+  for (int i = 1; i < L; ++i) {
+    if (i < nl) {
+      t = static_cast<u64>(w[i]) * m + (t >> 32);
+      w[i] = static_cast<uint32_t>(t);
+    }
+  }
 }
 
-__device__ __forceinline__ bool geq3(const u64 (&a)[3], const u64 (&b)[3]) {
-  if (a[2] != b[2]) return a[2] > b[2];
-  if (a[1] != b[1]) return a[1] > b[1];
-  return a[0] >= b[0];
-}
-
-__device__ __forceinline__ void sub3(const u64 (&a)[3], const u64 (&b)[3], u64 (&r)[3]) {
-  u64 r0 = a[0] - b[0];
-  u64 br = a[0] < b[0];
-  u64 t1 = a[1] - b[1];
-  u64 br1 = a[1] < b[1];
-  u64 r1 = t1 - br;
-  br1 |= t1 < br;
-  r[0] = r0;
-  r[1] = r1;
-  r[2] = a[2] - b[2] - br1;
-}
-
-__device__ __forceinline__ int bitlen3(const u64 (&x)[3]) {
-  if (x[2]) return 192 - __clzll(static_cast<long long>(x[2]));
-  if (x[1]) return 128 - __clzll(static_cast<long long>(x[1]));
-  if (x[0]) return 64 - __clzll(static_cast<long long>(x[0]));
-  return 0;
-}
-
-// `cnt` (≤ 64) bits of x starting at bit `pos` (pos ≥ 0).
-__device__ __forceinline__ u64 bits3(const u64 (&x)[3], int pos, int cnt) {
-  const int w = pos >> 6, b = pos & 63;
-  u64 lo = w < 3 ? x[w] : 0;
-  u64 hi = w + 1 < 3 ? x[w + 1] : 0;
-  u64 v = b ? (lo >> b) | (hi << (64 - b)) : lo;
-  return cnt >= 64 ? v : (v & ((1ull << cnt) - 1));
-}
-
-// Any bit of x below position pos (pos ≥ 0)?
-__device__ __forceinline__ bool sticky3(const u64 (&x)[3], int pos) {
-  if (pos <= 0) return false;
-  const int w = pos >> 6, b = pos & 63;
-  bool s = false;
-  for (int t = 0; t < 3 && t < w; ++t) s |= x[t] != 0;
-  if (w < 3 && b) s |= (x[w] & ((1ull << b) - 1)) != 0;
-  return s;
-}
-
-// Nearest double (ties to even) to (-1)^neg · mag · 2^E.
-__device__ __forceinline__ double round_to_double(const u64 (&mag)[3], int E, bool neg) {
-  const int L = bitlen3(mag);
+// Nearest double (ties to even) to (-1)^neg · (x + δ) · 2^E, where δ ∈ [0, 1)
+// is nonzero exactly when `sticky` is set (bits already shifted out of x).
+__device__ __forceinline__ double round_to_double(u64 x, bool sticky, int E, bool neg) {
   const u64 sign = neg ? (1ull << 63) : 0ull;
-  if (L == 0) return __longlong_as_double(static_cast<long long>(sign));
-  const int top = L - 1 + E;                     // exponent of the leading bit
+  if (x == 0) return __longlong_as_double(static_cast<long long>(sign));
+  const int Lb = 64 - __clzll(static_cast<long long>(x));
+  const int top = Lb - 1 + E;  // exponent of the leading bit
   if (top > 1023) return __longlong_as_double(static_cast<long long>(sign | 0x7FF0000000000000ull));
   const int p = top >= -1022 ? 53 : top + 1075;  // significant bits available
-  const int sh = L - p;                          // bits dropped (may be ≤ 0)
+  const int sh = Lb - p;                         // bits to drop (≤ 63)
   u64 q;
   if (sh <= 0) {
-    q = mag[0] << (-sh);                         // L ≤ 53: exact
+    q = x << (-sh);  // Lb ≤ p ≤ 53; no bits were shifted out (sticky implies Lb = 64)
   } else if (p <= 0) {
-    // Everything is below the last subnormal bit position + 1.
-    const bool above_half = (p == 0) && sticky3(mag, L - 1);  // mag > 2^(L-1) = half
-    q = above_half ? 1 : 0;
+    // Below the smallest subnormal: round up only when strictly above half of it.
+    const bool below = (x & ((1ull << (Lb - 1)) - 1)) != 0 || sticky;
+    q = (p == 0 && below) ? 1 : 0;
   } else {
-    q = bits3(mag, sh, p);
-    const bool rbit = bits3(mag, sh - 1, 1) != 0;
-    const bool st = sticky3(mag, sh - 1);
+    q = x >> sh;
+    const bool rbit = ((x >> (sh - 1)) & 1) != 0;
+    const bool st = sticky || (x & ((1ull << (sh - 1)) - 1)) != 0;
     if (rbit && (st || (q & 1))) ++q;
   }
   if (q == 0) return __longlong_as_double(static_cast<long long>(sign));
-  if (p < 53 || top < -1022) {
-    // Subnormal scale: value = q · 2^-1074 (q = 2^52 is the smallest normal).
-    return __longlong_as_double(static_cast<long long>(sign | q));
-  }
-  int f = top;                                   // q ∈ [2^52, 2^53]
+  if (p < 53) return __longlong_as_double(static_cast<long long>(sign | q));  // q · 2^-1074 (2^52: smallest normal)
+  int f = top;  // q ∈ [2^52, 2^53]
   if (q >> 53) {
     q >>= 1;
     ++f;
   }
   if (f > 1023) return __longlong_as_double(static_cast<long long>(sign | 0x7FF0000000000000ull));
-  const u64 bits = (static_cast<u64>(f + 1023) << 52) | (q & ((1ull << 52) - 1));
-  return __longlong_as_double(static_cast<long long>(sign | bits));
+  return __longlong_as_double(
+      static_cast<long long>(sign | (static_cast<u64>(f + 1023) << 52) | (q & ((1ull << 52) - 1))));
+}
+
+// (a·w) mod m for a < 2^32 and a fixed w < m with wp = ⌊w·2^32/m⌋ (V. Shoup's
+// modular multiplication with a precomputed quotient): q = ⌊a·wp/2^32⌋ is
+// the true quotient or one less, so a·w - q·m ∈ [0, 2m).
+__device__ __forceinline__ uint32_t mulmod_shoup(uint32_t a, uint32_t w, uint32_t wp, uint32_t m) {
+  const uint32_t q = __umulhi(a, wp);
+  const uint32_t r = a * w - q * m;
+  return r >= m ? r - m : r;
 }
 
 // One output: centred residues c[0..R) → nearest double of X·2^E.
 template <int R>
 __device__ __forceinline__ double crt_value(const int (&c)[R], int E, const Oz2Moduli& mods) {
   // Garner digits (Eq. garner): v_k = (c_k - Σ_{j<k} v_j P_{j-1}) P_{k-1}^{-1} mod m_k,
-  // with (P_{j-1} mod m_k) precomputed; goff_k (a multiple of m_k ≥ 2^27) keeps
-  // the 32-bit sum positive.
+  // with (P_{j-1} mod m_k) precomputed.  The sums are carried for every later
+  // modulus as soon as a digit is known, so each digit waits on one
+  // multiply-add; goff_k (a multiple of m_k ≥ 2^27) keeps them positive.
+  int S[R];
+#pragma unroll
+  for (int k = 0; k < R; ++k) S[k] = mods.goff[k] + c[k];
   uint32_t v[R];
 #pragma unroll
   for (int k = 0; k < R; ++k) {
-    int acc = mods.goff[k] + c[k];
+    v[k] = mulmod_shoup(static_cast<uint32_t>(S[k]), static_cast<uint32_t>(mods.inv[k]), mods.invp[k],
+                        static_cast<uint32_t>(mods.m[k]));
 #pragma unroll
-    for (int t = 0; t < k; ++t) acc -= static_cast<int>(v[t]) * mods.pmod[k][t];
-    const uint32_t mk = static_cast<uint32_t>(mods.m[k]);
-    const uint32_t t0 = mod_magic(static_cast<uint32_t>(acc), mk, mods.magic[k], mods.magic_sh[k]);
-    v[k] = mod_magic(t0 * static_cast<uint32_t>(mods.inv[k]), mk, mods.magic[k], mods.magic_sh[k]);
+    for (int j = k + 1; j < R; ++j) S[j] -= static_cast<int>(v[k]) * mods.pmod[j][k];
   }
-  // Mixed radix → integer by Horner from the top digit.  The top six digits
-  // stay below 2^61 (six moduli ≤ 1089), so they run in 64-bit arithmetic.
-  constexpr int H = R < 6 ? R : 6;
-  u64 top = v[R - 1];
+  // Mixed radix → integer by Horner from the top digit; after j steps the value
+  // is below the product of j+1 moduli < 2^(11(j+1)), which bounds the limbs.
+  constexpr int L = R <= 12 ? 4 : 5;  // M < 2^112 (r ≤ 12), < 2^148 (r ≤ 16)
+  uint32_t w[L];
+  w[0] = v[R - 1];
 #pragma unroll
-  for (int k = R - 2; k >= R - H; --k) top = top * static_cast<u32>(mods.m[k]) + v[k];
-  u64 X[3] = {top, 0, 0};
+  for (int i = 1; i < L; ++i) w[i] = 0;
 #pragma unroll
-  for (int k = R - H - 1; k >= 0; --k) mul_add(X, static_cast<uint32_t>(mods.m[k]), v[k], R > 12);
+  for (int k = R - 2; k >= 0; --k) {
+    const int nl = (11 * (R - k) + 31) / 32 < L ? (11 * (R - k) + 31) / 32 : L;
+    horner_step<L>(w, nl, static_cast<uint32_t>(mods.m[k]), v[k]);
+  }
   // Symmetric range [-M/2, M/2) (Eq. M-bound): X ≥ ⌈M/2⌉ ⇔ 2X ≥ M.
-  const bool neg = geq3(X, mods.Mhalf);
-  u64 mag[3];
-  if (neg) {
-    sub3(mods.M, X, mag);
-  } else {
-    mag[0] = X[0];
-    mag[1] = X[1];
-    mag[2] = X[2];
+  bool ge = true, decided = false;
+#pragma unroll
+  for (int i = L - 1; i >= 0; --i) {
+    const uint32_t h = static_cast<uint32_t>(mods.Mhalf[i >> 1] >> (32 * (i & 1)));
+    if (!decided && w[i] != h) {
+      ge = w[i] > h;
+      decided = true;
+    }
   }
-  return round_to_double(mag, E, neg);
+  const bool neg = ge;
+  if (neg) {  // |X - M| = M - X
+    uint32_t borrow = 0;
+#pragma unroll
+    for (int i = 0; i < L; ++i) {
+      const u64 t = static_cast<u64>(static_cast<uint32_t>(mods.M[i >> 1] >> (32 * (i & 1)))) - w[i] - borrow;
+      w[i] = static_cast<uint32_t>(t);
+      borrow = static_cast<uint32_t>(t >> 63);
+    }
+  }
+  // Leading 64 bits and a sticky bit for everything below them.
+  u128 x = (static_cast<u128>(w[3]) << 96) | (static_cast<u128>(w[2]) << 64) | (static_cast<u128>(w[1]) << 32) | w[0];
+  bool sticky = false;
+  if (L == 5 && w[L - 1] != 0) {
+    sticky = w[0] != 0;
+    x = (static_cast<u128>(w[L - 1]) << 96) | (x >> 32);
+    E += 32;
+  }
+  const u64 xh = static_cast<u64>(x >> 64);
+  u64 top64 = static_cast<u64>(x);
+  if (xh) {
+    const int s = 64 - __clzll(static_cast<long long>(xh));  // bits above the low word
+    top64 = (xh << (64 - s)) | (static_cast<u64>(x) >> s);
+    sticky = sticky || (static_cast<u64>(x) << (64 - s)) != 0;
+    E += s;
+  }
+  return round_to_double(top64, sticky, E, neg);
 }
 
-// Four consecutive rows of one column per thread: 8-byte residue loads per
-// modulus (int16 × 4) and two 16-byte stores of C when the layout allows.
-// The four outputs are computed one after the other (not interleaved) to keep
-// the register footprint of the r-deep Garner recurrence small.
 template <int R>
-__global__ void __launch_bounds__(256) crt_kernel(int64_t m, int64_t n, const __grid_constant__ Oz2Moduli mods,
-                                                  const int16_t* __restrict__ res, int64_t ldr,
-                                                  const int* __restrict__ d, const int* __restrict__ e,
-                                                  double* __restrict__ C, int64_t ldc, int vec_in, int vec_out) {
-  const int64_t i0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) * 4;
-  if (i0 >= m) return;
-  const bool full = i0 + 3 < m;
-  const size_t mstride = static_cast<size_t>(ldr) * n;
-  int di[4];
+__global__ void __launch_bounds__(kCrtThreads) crt_kernel(int64_t m, int64_t n, const __grid_constant__ Oz2Moduli mods,
+                                                          const int16_t* __restrict__ res, int64_t ldr,
+                                                          const int* __restrict__ d, const int* __restrict__ e,
+                                                          double* __restrict__ C, int64_t ldc, int vec_in) {
+  __shared__ double tile[kCrtRows][kCrtCols + 1];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t tiles_m = static_cast<uint32_t>((m + kCrtRows - 1) / kCrtRows);
+  const uint32_t ntiles = tiles_m * static_cast<uint32_t>((n + kCrtCols - 1) / kCrtCols);
+  const size_t mstride = static_cast<size_t>(m) * ldr;
+  for (uint32_t t = blockIdx.x; t < ntiles; t += gridDim.x) {
+    const int64_t r0 = static_cast<int64_t>(t % tiles_m) * kCrtRows, c0 = static_cast<int64_t>(t / tiles_m) * kCrtCols;
+    const int64_t cb = c0 + 4 * lane;
+    int ecol[4];
 #pragma unroll
-  for (int u = 0; u < 4; ++u) di[u] = i0 + u < m ? d[i0 + u] : 0;
-  for (int64_t j = blockIdx.y; j < n; j += gridDim.y) {
-    const int16_t* p = res + j * ldr + i0;
-    uint32_t lo[R], hi[R];   // residues of rows (i0, i0+1) and (i0+2, i0+3), packed int16 pairs
-    if (vec_in && full) {
+    for (int u = 0; u < 4; ++u) ecol[u] = cb + u < n ? e[cb + u] : 0;
+    for (int s = 0; s < kCrtRows / 8; ++s) {
+      const int lr = warp + 8 * s;
+      const int64_t row = r0 + lr;
+      if (row >= m) continue;
+      const int dr = d[row];
+      const int16_t* p = res + row * ldr + cb;
+      uint32_t lo[R], hi[R];  // residues of columns (cb, cb+1) and (cb+2, cb+3), packed int16 pairs
+      if (vec_in && cb + 3 < n) {
 #pragma unroll
-      for (int k = 0; k < R; ++k) {
-        const uint2 q = __ldg(reinterpret_cast<const uint2*>(p + k * mstride));
-        lo[k] = q.x;
-        hi[k] = q.y;
+        for (int k = 0; k < R; ++k) {
+          const uint2 q = __ldg(reinterpret_cast<const uint2*>(p + k * mstride));
+          lo[k] = q.x;
+          hi[k] = q.y;
+        }
+      } else {
+#pragma unroll
+        for (int k = 0; k < R; ++k) {
+          uint32_t w4[4];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) w4[u] = cb + u < n ? static_cast<uint16_t>(p[k * mstride + u]) : 0u;
+          lo[k] = w4[0] | (w4[1] << 16);
+          hi[k] = w4[2] | (w4[3] << 16);
+        }
       }
-    } else {
-#pragma unroll
-      for (int k = 0; k < R; ++k) {
-        uint32_t w[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) w[u] = i0 + u < m ? static_cast<uint16_t>(p[k * mstride + u]) : 0u;
-        lo[k] = w[0] | (w[1] << 16);
-        hi[k] = w[2] | (w[3] << 16);
-      }
-    }
-    const int ej = e[j];
-    double2 o01, o23;
 #pragma unroll 1
-    for (int u = 0; u < 4; ++u) {
-      int c[R];
+      for (int u = 0; u < 4; ++u) {
+        int c[R];
 #pragma unroll
-      for (int k = 0; k < R; ++k) {
-        const uint32_t w = u < 2 ? lo[k] : hi[k];
-        c[k] = static_cast<int>(static_cast<int16_t>((u & 1) ? (w >> 16) : (w & 0xFFFFu)));
+        for (int k = 0; k < R; ++k) {
+          const uint32_t w = u < 2 ? lo[k] : hi[k];
+          c[k] = static_cast<int>(static_cast<int16_t>((u & 1) ? (w >> 16) : (w & 0xFFFFu)));
+        }
+        const int eu = u == 0 ? ecol[0] : u == 1 ? ecol[1] : u == 2 ? ecol[2] : ecol[3];
+        tile[lr][4 * lane + u] = crt_value<R>(c, -(dr + eu), mods);
       }
-      const int du = u == 0 ? di[0] : u == 1 ? di[1] : u == 2 ? di[2] : di[3];
-      const double val = crt_value<R>(c, -(du + ej), mods);
-      if (u == 0) o01.x = val;
-      else if (u == 1) o01.y = val;
-      else if (u == 2) o23.x = val;
-      else o23.y = val;
     }
-    double* q = C + i0 + j * ldc;
-    if (vec_out && full) {
-      reinterpret_cast<double2*>(q)[0] = o01;
-      reinterpret_cast<double2*>(q)[1] = o23;
-    } else {
-      const double out[4] = {o01.x, o01.y, o23.x, o23.y};
-#pragma unroll
-      for (int u = 0; u < 4; ++u)
-        if (i0 + u < m) q[u] = out[u];
+    __syncthreads();
+    // Column segments of 32 rows (256 bytes) per warp.
+    const int64_t row = r0 + lane;
+    for (int cc = warp; cc < kCrtCols; cc += kCrtThreads / 32) {
+      const int64_t col = c0 + cc;
+      if (col < n && row < m) C[row + col * ldc] = tile[lane][cc];
     }
+    __syncthreads();
   }
 }
 
 template <int R>
-static void launch_crt_r(dim3 g, cudaStream_t st, int64_t m, int64_t n, const Oz2Moduli& mods, const int16_t* res,
-                         int64_t ldr, const int32_t* d, const int32_t* e, double* C, int64_t ldc, int vi, int vo) {
-  crt_kernel<R><<<g, 256, 0, st>>>(m, n, mods, res, ldr, d, e, C, ldc, vi, vo);
+static void launch_crt_r(int grid, cudaStream_t st, int64_t m, int64_t n, const Oz2Moduli& mods, const int16_t* res,
+                         int64_t ldr, const int32_t* d, const int32_t* e, double* C, int64_t ldc, int vi) {
+  crt_kernel<R><<<grid, kCrtThreads, 0, st>>>(m, n, mods, res, ldr, d, e, C, ldc, vi);
 }
 
 cudaError_t launch_reconstruct(int64_t m, int64_t n, const Oz2Moduli& mods, const int16_t* residues,
                                int64_t ldr, const int32_t* d, const int32_t* e, double* C, int64_t ldc,
                                cudaStream_t st) {
   if (m == 0 || n == 0) return cudaSuccess;
-  dim3 g(static_cast<unsigned>((m + 1023) / 1024), static_cast<unsigned>(n < 65535 ? n : 65535));
+  const int64_t tiles = ((m + kCrtRows - 1) / kCrtRows) * ((n + kCrtCols - 1) / kCrtCols);
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int grid = static_cast<int>(tiles < 16LL * sms ? tiles : 16LL * sms);
   const int vi = (ldr % 4 == 0) && (reinterpret_cast<uintptr_t>(residues) % 8 == 0);
-  const int vo = (ldc % 2 == 0) && (reinterpret_cast<uintptr_t>(C) % 16 == 0);
   count_launch();
   switch (mods.r) {
 #define OZ2_CRT_CASE(R) \
   case R:               \
-    launch_crt_r<R>(g, st, m, n, mods, residues, ldr, d, e, C, ldc, vi, vo); \
+    launch_crt_r<R>(grid, st, m, n, mods, residues, ldr, d, e, C, ldc, vi); \
     break;
     OZ2_CRT_CASE(1) OZ2_CRT_CASE(2) OZ2_CRT_CASE(3) OZ2_CRT_CASE(4) OZ2_CRT_CASE(5) OZ2_CRT_CASE(6)
     OZ2_CRT_CASE(7) OZ2_CRT_CASE(8) OZ2_CRT_CASE(9) OZ2_CRT_CASE(10) OZ2_CRT_CASE(11) OZ2_CRT_CASE(12)

@@ -17,14 +17,15 @@
 // accumulator merge of §2.5 "Accumulators").  Every K-slab (32768 squares,
 // 4096 nonsquare: Eq. accum-exact) the epilogue reads the accumulators and
 // forms  v = acc0 + s·acc1  or  v = 16·acc0 - 15·acc1  mod m, adds the
-// previous slab's residue and stores the centred residue as int16.
+// previous slab's residue and stores the centred residue as int16, row-major
+// (each thread owns one row and 16 consecutive columns: 16-byte stores).
 //
 // Pipeline: a stage is one (A plane, B plane) pair of 128-byte-deep tiles
 // (32 KiB per CTA), six stages.  Warp 0 of each CTA issues its CTA's TMA
 // loads, completing on the leader's stage barrier; warp 1 of the leader
 // issues the MMAs and multicasts stage releases and accumulator-ready
-// signals to both CTAs; warps 2..9 of both CTAs run the epilogue and release
-// the accumulators to the leader.  Every wait is bounded; on expiry the
+// signals to both CTAs; warps 2..17 of both CTAs run the epilogue (64
+// columns each) and release the accumulators to the leader.  Every wait is bounded; on expiry the
 // kernel records OZ2_ERR_TIMEOUT in the device status word and drains.
 #include <algorithm>
 
@@ -38,45 +39,54 @@ constexpr int kBK = 128;                         // k-bytes per stage
 constexpr int kTileBytes = kRows * kBK;          // 16 KiB
 constexpr int kStageBytes = 2 * kTileBytes;      // A tile + B tile
 constexpr int kStages = 6;
-constexpr int kGemmThreads = 320;                // 10 warps
-constexpr int kEpiWarps = 8;
+constexpr int kEpiWarps = 16;
+constexpr int kGemmThreads = 32 * (2 + kEpiWarps);  // producer, MMA, epilogue
 constexpr int kTmemCols = 512;
 constexpr int kAccCols = 256;
 constexpr int kGroupM = 8;                       // tile rasterisation group
 constexpr long long kWaitLimit = 4000000000LL;   // ≈2 s at 2 GHz
 
 // ---- epilogue arithmetic shared by the tensor-core and SIMT kernels --------
-// x - m·rint(x/m) for an exactly represented integer |x| < 2^24: the FMA
-// forms x - q·m exactly, and q is within one of x/m, so |result| < 1.5m.
+// All on the FMA pipe.  Rounding to an integer uses the 1.5·2^23 constant:
+// for |y| < 2^22, fl(y + 1.5·2^23) - 1.5·2^23 = round-to-nearest(y), and the
+// low 16 bits of the sum's encoding are that integer in two's complement.
+constexpr float kRoundMagic = 12582912.f;  // 1.5·2^23
+
+// x - m·round(x/m) for an exactly represented integer |x| ≤ 2^24: the FMA
+// forms x - q·m exactly and q is within one of x/m, so |result| < 1.5m.
 __device__ __forceinline__ float loose_mod(float x, float m, float inv_m) {
-  float q = rintf(x * inv_m);
+  const float q = fmaf(x, inv_m, kRoundMagic) - kRoundMagic;
   return fmaf(-q, m, x);
 }
-// Centred representative in [-⌊m/2⌋, m-1-⌊m/2⌋] of an integer |x| < 2^24.
-__device__ __forceinline__ int centred_mod(float x, float m, float inv_m, int lo, int hi) {
-  int r = static_cast<int>(loose_mod(x, m, inv_m));
-  const int mi = static_cast<int>(m);
-  if (r > hi) r -= mi;
-  if (r < lo) r += mi;
-  if (r > hi) r -= mi;
-  if (r < lo) r += mi;
-  return r;
+// Centred representative in [-⌊m/2⌋, m-1-⌊m/2⌋] of an integer |v| < 2^16:
+// here v/m is off by under 2^-14 and lies ≥ 1/(2m) > 2^-12 from every
+// half-integer unless v/m is one (even m), so the rounding is exact and only
+// the tie +m/2 needs moving to -m/2.
+__device__ __forceinline__ float centred_small(float v, float m, float inv_m, float hi) {
+  const float q = fmaf(v, inv_m, kRoundMagic) - kRoundMagic;
+  const float r = fmaf(-q, m, v);
+  return r > hi ? r - m : r;
 }
 // Recombine one element's two accumulators (Eq. sq-shortcut, or Eq. kar with
 // the merged accumulator), add the previous slab's residue, and reduce.
-__device__ __forceinline__ int combine_residue(float a0, float a1, bool square, float s, float m, float inv_m,
-                                               int lo, int hi, int prev) {
+__device__ __forceinline__ float combine_residue(float a0, float a1, bool square, float s, float m, float inv_m,
+                                                 float hi, float prev) {
   const float r0 = loose_mod(a0, m, inv_m);
   const float r1 = loose_mod(a1, m, inv_m);
   // square: d0e0 + s(d1e0 + d0e1), |v| < 2^16
   // nonsquare (b = 4): 2^b Σ + (1-2^b)(d0e0 - 2^b d1e1), |v| < 2^15
-  float v = square ? fmaf(s, r1, r0) : fmaf(16.f, r0, -15.f * r1);
-  v += static_cast<float>(prev);
-  return centred_mod(v, m, inv_m, lo, hi);
+  const float v = (square ? fmaf(s, r1, r0) : fmaf(16.f, r0, -15.f * r1)) + prev;
+  return centred_small(v, m, inv_m, hi);
+}
+// int16 encoding of an integer-valued float in [-2^15, 2^15).
+__device__ __forceinline__ uint32_t as_i16_bits(float r) { return __float_as_uint(r + kRoundMagic) & 0xFFFFu; }
+__device__ __forceinline__ float i16_to_float(uint32_t bits16) {
+  return __uint_as_float(0x4B400000u + static_cast<uint32_t>(static_cast<int>(static_cast<int16_t>(bits16)))) -
+         kRoundMagic;
 }
 
 struct EpiCtx {
-  int16_t* res;   // r × (m×n, ld = m)
+  int16_t* res;   // r × (m×n row-major, ld = n)
   float* urow;
   Oz2Device* dev;
   int64_t m, n;
@@ -262,25 +272,25 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     }
     __syncwarp();
   } else {
-    // ---------------- epilogue (warps 2..9, both CTAs) ----------------
+    // ---------------- epilogue (warps 2..17, both CTAs) ----------------
     const int q = warp & 3;                    // TMEM lane quarter of this warp
-    const int h = (warp - 2) >> 2;             // column half
-    const uint32_t lane_addr = tmem + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(128 * h);
+    const int h = (warp - 2) >> 2;             // 64-column quarter of the tile
+    const uint32_t lane_addr = tmem + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(64 * h);
     const uint32_t acc_empty_leader = mapa_shared(acc_empty, 0);
+    const bool vec_ok = (ctx.n % 8) == 0;
     uint32_t accph = 0;
     for (int64_t u = pair; u < um.nunits && ok; u += npairs) {
       int i;
       int64_t tm, tn;
       unit_coords(u, um, &i, &tm, &tn);
       const int64_t row = tm * kTileM + rank * kRows + 32 * q + lane;
-      const int64_t col0 = tn * kTileN + 128 * h;
+      const int64_t col0 = tn * kTileN + 64 * h;
       const bool square = MODE == 0 ? mods.sq_base[i] != 0 : true;
       const float mf = MODE == 0 ? static_cast<float>(mods.m[i]) : 1.f;
       const float inv = 1.f / mf;
       const float sb = MODE == 0 ? static_cast<float>(mods.sq_base[i]) : 0.f;
-      const int lo = MODE == 0 ? -(mods.m[i] / 2) : 0;
-      const int hi = MODE == 0 ? mods.m[i] - 1 - mods.m[i] / 2 : 0;
-      int16_t* resi = MODE == 0 ? ctx.res + static_cast<size_t>(i) * ctx.m * ctx.n : nullptr;
+      const float hi = MODE == 0 ? static_cast<float>(mods.m[i] - 1 - mods.m[i] / 2) : 0.f;
+      int16_t* rrow = MODE == 0 ? ctx.res + static_cast<size_t>(i) * ctx.m * ctx.n + row * ctx.n : nullptr;
       const int64_t slab = slab_steps_of<MODE>(mods, i, ksteps);
       float rowmax = 0.f;
       for (int64_t kb0 = 0; kb0 < ksteps; kb0 += slab) {
@@ -289,23 +299,58 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           break;
         }
         tc_fence_after();
-        for (int c = 0; c < 128; c += 32) {
-          uint32_t v0[32], v1[32];
-          tmem_ld32(lane_addr + c, v0);
-          if (MODE == 0) tmem_ld32(lane_addr + kAccCols + c, v1);
+        for (int c = 0; c < 64; c += 16) {
+          uint32_t v0[16], v1[16];
+          tmem_ld16(lane_addr + c, v0);
+          if (MODE == 0) tmem_ld16(lane_addr + kAccCols + c, v1);
           tmem_ld_wait();
           if (MODE == 1) {
 #pragma unroll
-            for (int j = 0; j < 32; ++j) rowmax = fmaxf(rowmax, __uint_as_float(v0[j]));
+            for (int j = 0; j < 16; ++j) rowmax = fmaxf(rowmax, __uint_as_float(v0[j]));
           } else if (row < ctx.m) {
+            const int64_t cc = col0 + c;
+            int16_t* dst = rrow + cc;
+            const bool full = vec_ok && cc + 16 <= ctx.n;
+            uint32_t prevw[8];
+            if (kb0 && full) {
 #pragma unroll
-            for (int j = 0; j < 32; ++j) {
-              const int64_t col = col0 + c + j;
-              if (col < ctx.n) {
-                int16_t* dst = resi + col * ctx.m + row;
-                const int prev = kb0 ? *dst : 0;
-                *dst = static_cast<int16_t>(combine_residue(__uint_as_float(v0[j]), __uint_as_float(v1[j]), square,
-                                                            sb, mf, inv, lo, hi, prev));
+              for (int t = 0; t < 2; ++t) {
+                const uint4 pv = reinterpret_cast<const uint4*>(dst)[t];
+                prevw[4 * t] = pv.x;
+                prevw[4 * t + 1] = pv.y;
+                prevw[4 * t + 2] = pv.z;
+                prevw[4 * t + 3] = pv.w;
+              }
+            } else {
+#pragma unroll
+              for (int t = 0; t < 8; ++t) {
+                uint32_t a = 0, b = 0;
+                if (kb0 && cc + 2 * t < ctx.n) a = static_cast<uint16_t>(dst[2 * t]);
+                if (kb0 && cc + 2 * t + 1 < ctx.n) b = static_cast<uint16_t>(dst[2 * t + 1]);
+                prevw[t] = a | (b << 16);
+              }
+            }
+            uint32_t outw[8];
+#pragma unroll
+            for (int t = 0; t < 8; ++t) {
+              const float p0 = kb0 ? i16_to_float(prevw[t] & 0xFFFFu) : 0.f;
+              const float p1 = kb0 ? i16_to_float(prevw[t] >> 16) : 0.f;
+              const float r0 = combine_residue(__uint_as_float(v0[2 * t]), __uint_as_float(v1[2 * t]), square, sb, mf,
+                                               inv, hi, p0);
+              const float r1 = combine_residue(__uint_as_float(v0[2 * t + 1]), __uint_as_float(v1[2 * t + 1]), square,
+                                               sb, mf, inv, hi, p1);
+              outw[t] = as_i16_bits(r0) | (as_i16_bits(r1) << 16);
+            }
+            if (full) {
+#pragma unroll
+              for (int t = 0; t < 2; ++t)
+                reinterpret_cast<uint4*>(dst)[t] =
+                    make_uint4(outw[4 * t], outw[4 * t + 1], outw[4 * t + 2], outw[4 * t + 3]);
+            } else {
+#pragma unroll
+              for (int t = 0; t < 8; ++t) {
+                if (cc + 2 * t < ctx.n) dst[2 * t] = static_cast<int16_t>(outw[t] & 0xFFFFu);
+                if (cc + 2 * t + 1 < ctx.n) dst[2 * t + 1] = static_cast<int16_t>(outw[t] >> 16);
               }
             }
           }
@@ -364,10 +409,10 @@ __global__ void plane_gemm_simt_kernel(const uint8_t* __restrict__ pa, const uin
     const bool square = mods.sq_base[i] != 0;
     const float mf = static_cast<float>(mods.m[i]);
     const float inv = 1.f / mf;
-    const int lo = -(mods.m[i] / 2), hi = mods.m[i] - 1 - mods.m[i] / 2;
+    const float hi = static_cast<float>(mods.m[i] - 1 - mods.m[i] / 2);
     const size_t p0 = mods.plane_off[i];
     const int64_t slab = square ? kKSlabSquare : kKSlabMerged;
-    int res = 0;
+    float res = 0.f;
     for (int64_t l0 = 0; l0 < k_pad; l0 += slab) {
       float a0 = 0.f, a1 = 0.f;
       const int64_t l1 = min(k_pad, l0 + slab);
@@ -383,9 +428,9 @@ __global__ void plane_gemm_simt_kernel(const uint8_t* __restrict__ pa, const uin
           a1 += x1 * y1 + x2 * y2;
         }
       }
-      res = combine_residue(a0, a1, square, static_cast<float>(mods.sq_base[i]), mf, inv, lo, hi, res);
+      res = combine_residue(a0, a1, square, static_cast<float>(mods.sq_base[i]), mf, inv, hi, res);
     }
-    ctx.res[static_cast<size_t>(i) * ctx.m * ctx.n + col * ctx.m + row] = static_cast<int16_t>(res);
+    ctx.res[static_cast<size_t>(i) * ctx.m * ctx.n + row * ctx.n + col] = static_cast<int16_t>(res);
   }
 }
 

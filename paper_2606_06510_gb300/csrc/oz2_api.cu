@@ -149,6 +149,7 @@ static Oz2Moduli build_moduli(int r, int quant) {
       P = (P * kModuliAll[t]) % m;
     }
     c.inv[i] = i ? mod_inverse(P, m) : 1;
+    c.invp[i] = static_cast<uint32_t>((static_cast<u64>(c.inv[i]) << 32) / static_cast<u64>(m));
   }
   c.nplanes = plane;
   c.table_entries = toff;
@@ -422,7 +423,7 @@ int oz2_dgemm_ex(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, 
   if (err == cudaSuccess)
     err = launch_plane_gemm(m, n, L.k_pad, mods, pa, pb, simt ? 2 : 0, res, nullptr, ds->status, s);
   mark(6);
-  if (err == cudaSuccess) err = launch_reconstruct(m, n, mods, res, m, d, e, C, ldc, s);
+  if (err == cudaSuccess) err = launch_reconstruct(m, n, mods, res, n, d, e, C, ldc, s);
   mark(7);
   if (err == cudaSuccess) err = launch_fallback_lists(m, n, k, A, lda, B, ldb, rf, cf, misc, C, ldc, s);
   mark(8);
@@ -631,7 +632,7 @@ int oz2_residue_gemm_simt(int64_t m, int64_t n, int64_t k, int num_moduli, const
 
 int oz2_reconstruct(int64_t m, int64_t n, int num_moduli, const int16_t* residues, int64_t ldr, const int32_t* d,
                     const int32_t* e, double* C, int64_t ldc, void* stream) {
-  if (m < 0 || n < 0 || ldr < std::max<int64_t>(1, m) || ldc < std::max<int64_t>(1, m)) return OZ2_ERR_INVALID_ARG;
+  if (m < 0 || n < 0 || ldr < std::max<int64_t>(1, n) || ldc < std::max<int64_t>(1, m)) return OZ2_ERR_INVALID_ARG;
   if (num_moduli < 1 || num_moduli > kMaxModuli) return OZ2_ERR_UNSUPPORTED_R;
   if (m && n && (!residues || !d || !e || !C)) return OZ2_ERR_INVALID_ARG;
   const Oz2Moduli mods = build_moduli(num_moduli, OZ2_QUANT_TZ);
