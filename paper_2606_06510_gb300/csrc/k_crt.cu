@@ -4,6 +4,11 @@
 // (round-to-nearest-even) conversion of X·2^-(d_i+e_j) to FP64, including
 // the subnormal range.
 //
+// The reconstruction is computed by the direct CRT sum with a fixed-point
+// quotient (multiply-adds only); Garner's algorithm, the paper's method,
+// takes over in the rare case where that quotient is ambiguous, so every
+// output equals the Garner result exactly.
+//
 // Residues arrive row-major (r matrices of m×n, ld = ldr ≥ n) from the
 // residue GEMM; C is column-major.  A block computes a 32-row × 128-column
 // tile: each thread reads four consecutive residues of one row per modulus
@@ -146,6 +151,76 @@ __device__ __forceinline__ double crt_value(const int (&c)[R], int E, const Oz2M
   return round_to_double(top64, sticky, E, neg);
 }
 
+// Fast path: the same X by the direct CRT sum.  With u_k = c_k + coff_k ≥ 0,
+// S = Σ_k u_k W_k ≡ X (mod M), and S/M = Σ_k u_k y_k/m_k, so
+// q = ⌊S/M + 1/2⌋ gives X = S - q·M ∈ [-M/2, M/2).  q comes from the
+// 32.32 fixed-point sum Σ u_k F_k + 2^31, whose error is below
+// Σ u_k·2^-33 < 2^-13.3; when its fraction is within 2^19/2^32 of an integer
+// (X within that margin of ±M/2, which products bounded by Eq. M-bound never
+// reach) the caller falls back to Garner.  Returns false in that case.
+template <int R>
+__device__ __forceinline__ bool crt_value_fast(const int (&c)[R], int E, const Oz2Moduli& mods, double& out) {
+  constexpr int LW = R <= 12 ? 4 : 5;  // limbs of W_k (< M)
+  constexpr int LS = LW + 1;           // limbs of S (u_k < 2^16.1, r ≤ 16)
+  u64 acc[LS];
+#pragma unroll
+  for (int j = 0; j < LS; ++j) acc[j] = 0;
+  u64 Q = 1ull << 31;
+#pragma unroll
+  for (int k = 0; k < R; ++k) {
+    const uint32_t u = static_cast<uint32_t>(c[k] + mods.coff[k]);
+#pragma unroll
+    for (int j = 0; j < LW; ++j) acc[j] += static_cast<u64>(u) * mods.crtw[k][j];
+    Q += static_cast<u64>(u) * mods.crtf[k];
+  }
+  const uint32_t frac = static_cast<uint32_t>(Q);
+  if (frac < (1u << 19) || frac > 0xFFFFFFFFu - (1u << 19)) return false;
+  const uint32_t q = static_cast<uint32_t>(Q >> 32);
+  // x = S - q·M, two's complement over LS limbs.
+  uint32_t x[LS];
+  u64 sc = 0, pc = 0;
+  uint32_t borrow = 0;
+#pragma unroll
+  for (int j = 0; j < LS; ++j) {
+    const u64 sj = acc[j] + sc;
+    sc = sj >> 32;
+    const uint32_t mj = j < 6 ? static_cast<uint32_t>(mods.M[j >> 1] >> (32 * (j & 1))) : 0u;
+    const u64 pj = static_cast<u64>(q) * mj + pc;
+    pc = pj >> 32;
+    const u64 dj = static_cast<u64>(static_cast<uint32_t>(sj)) - static_cast<uint32_t>(pj) - borrow;
+    x[j] = static_cast<uint32_t>(dj);
+    borrow = static_cast<uint32_t>(dj >> 63);
+  }
+  const bool neg = (x[LS - 1] >> 31) != 0;
+  if (neg) {  // magnitude of the two's complement value
+    uint32_t cy = 1;
+#pragma unroll
+    for (int j = 0; j < LS; ++j) {
+      const u64 t = static_cast<u64>(~x[j]) + cy;
+      x[j] = static_cast<uint32_t>(t);
+      cy = static_cast<uint32_t>(t >> 32);
+    }
+  }
+  // |X| < M/2 fits in LW limbs; leading 64 bits and a sticky bit.
+  u128 v = (static_cast<u128>(x[3]) << 96) | (static_cast<u128>(x[2]) << 64) | (static_cast<u128>(x[1]) << 32) | x[0];
+  bool sticky = false;
+  if (LW == 5 && x[LW - 1] != 0) {
+    sticky = x[0] != 0;
+    v = (static_cast<u128>(x[LW - 1]) << 96) | (v >> 32);
+    E += 32;
+  }
+  const u64 vh = static_cast<u64>(v >> 64);
+  u64 top64 = static_cast<u64>(v);
+  if (vh) {
+    const int s = 64 - __clzll(static_cast<long long>(vh));
+    top64 = (vh << (64 - s)) | (static_cast<u64>(v) >> s);
+    sticky = sticky || (static_cast<u64>(v) << (64 - s)) != 0;
+    E += s;
+  }
+  out = round_to_double(top64, sticky, E, neg);
+  return true;
+}
+
 template <int R>
 __global__ void __launch_bounds__(kCrtThreads) crt_kernel(int64_t m, int64_t n, const __grid_constant__ Oz2Moduli mods,
                                                           const int16_t* __restrict__ res, int64_t ldr,
@@ -195,7 +270,9 @@ __global__ void __launch_bounds__(kCrtThreads) crt_kernel(int64_t m, int64_t n, 
           c[k] = static_cast<int>(static_cast<int16_t>((u & 1) ? (w >> 16) : (w & 0xFFFFu)));
         }
         const int eu = u == 0 ? ecol[0] : u == 1 ? ecol[1] : u == 2 ? ecol[2] : ecol[3];
-        tile[lr][4 * lane + u] = crt_value<R>(c, -(dr + eu), mods);
+        double val;
+        if (!crt_value_fast<R>(c, -(dr + eu), mods, val)) val = crt_value<R>(c, -(dr + eu), mods);
+        tile[lr][4 * lane + u] = val;
       }
     }
     __syncthreads();

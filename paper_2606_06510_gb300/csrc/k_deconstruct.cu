@@ -1,19 +1,25 @@
 // Deconstruction (Algorithm 1 "lin:quant" and "lin:dec"; §2.5 digit planes)
 // and the magnitude planes of the "+1" pass (§2.4).
 //
-// One thread handles 16 consecutive k-entries of one row of the operand
-// (a row of A, or a column of B seen as a row of Bᵀ); the two threads of a
-// lane pair cover 32 consecutive k-entries, so every plane row segment they
-// write is one full 32-byte sector (16-byte vector stores).  A is column-
-// major, so for A the 16 row-threads of a warp read 16 consecutive rows of
-// one column per load (coalesced); B's rows are contiguous in k.
+// One thread handles 8 consecutive k-entries of one row of the operand (a row
+// of A, or a column of B seen as a row of Bᵀ); the four threads of a lane
+// quad cover 32 consecutive k-entries, so every plane row segment they write
+// is one full 32-byte sector (8-byte stores per thread).  A is column-major:
+// a warp's 8 row-quads read 8 consecutive rows of 4 columns per load.  B's
+// rows are contiguous in k and are read with 16-byte vector loads.  One
+// launch covers both operands: the first blocks work on A, the rest on B.
+#include <algorithm>
+#include <utility>
+
 #include "oz2_common.cuh"
 
 namespace oz2 {
 
-constexpr int kElems = 16;               // k-entries per thread
-constexpr int kRowsPerBlock = 128;       // 256 threads = 128 rows × 2 halves
+constexpr int kElems = 8;                // k-entries per thread
+constexpr int kQuad = 4;                 // threads per 32-entry row segment
+constexpr int kSeg = kElems * kQuad;     // k-entries per tile column
 constexpr int kDecThreads = 256;
+constexpr int kRowsPerBlock = kDecThreads / kQuad;  // 64
 
 // Integer significand M and exponent x with |x| = M·2^x (M < 2^53), or M = 0.
 struct Split {
@@ -86,110 +92,149 @@ struct OperandView {
   const int32_t* exps;  // ra/cb (magnitude) or d/e (deconstruction)
   const uint8_t* flag;
   uint8_t* out;         // planes: rows × k_pad per plane
+  const uint32_t* table;  // packed digit planes per residue (deconstruction)
+  int vec;              // k contiguous and rows 16-byte aligned: vector loads
 };
 
-// MODE 0: magnitude plane (1 plane); MODE 1: residue digit planes.
-template <int MODE>
-__global__ void __launch_bounds__(kDecThreads) planes_kernel(OperandView X, int64_t k, int64_t k_pad,
-                                                             int clamp_c, int rn,
-                                                             const __grid_constant__ Oz2Moduli mods,
-                                                             const uint32_t* __restrict__ table_g) {
+// The 8 entries [l0, l0+8) of one row (zero beyond k).
+__device__ __forceinline__ void load8(const OperandView& X, int64_t row, int64_t l0, int64_t k, double (&x)[kElems]) {
+  const double* p = X.base + row * X.row_stride + l0 * X.k_stride;
+  if (X.vec && l0 + kElems <= k) {
+#pragma unroll
+    for (int t = 0; t < kElems / 2; ++t) {
+      const double2 v = __ldg(reinterpret_cast<const double2*>(p) + t);
+      x[2 * t] = v.x;
+      x[2 * t + 1] = v.y;
+    }
+  } else {
+#pragma unroll
+    for (int e = 0; e < kElems; ++e) x[e] = l0 + e < k ? __ldg(p + e * X.k_stride) : 0.0;
+  }
+}
+
+// Residues of 8 entries modulo modulus I and their E4M3 digit planes (the
+// modulus's constants are compile-time constants).
+template <int I>
+__device__ __forceinline__ void planes_one(const uint32_t (&u0)[kElems], const uint32_t (&u1)[kElems],
+                                           const uint32_t (&u2)[kElems], const uint32_t (&u3)[kElems],
+                                           const uint32_t (&ng)[kElems], const uint32_t* table, uint8_t* dst,
+                                           size_t plane_stride) {
+  constexpr ModConst mc = mod_const(I);
+  uint32_t w[kElems];
+#pragma unroll
+  for (int e = 0; e < kElems; ++e) {
+    // Ã mod m from the limbs: u0 + u1·2^16 + u2·2^32 + u3·2^48 - ng·2^64 (mod m), < 2^28
+    const uint32_t y = u0[e] + u1[e] * mc.limb1 + u2[e] * mc.limb2 + u3[e] * mc.limb3 + ng[e] * mc.neg64;
+    w[e] = table[mc.table_off + mod_magic(y, mc.m, mc.magic, mc.sh)];  // packed E4M3 planes of centred(r)
+  }
+  uint8_t* pdst = dst + static_cast<size_t>(mc.plane_off) * plane_stride;
+#pragma unroll
+  for (int p = 0; p < (mc.s ? 2 : 3); ++p)
+    *reinterpret_cast<uint2*>(pdst + p * plane_stride) =
+        make_uint2(gather_byte(w[0], w[1], w[2], w[3], p), gather_byte(w[4], w[5], w[6], w[7], p));
+}
+
+template <int... Is>
+__device__ __forceinline__ void planes_all(std::integer_sequence<int, Is...>, const uint32_t (&u0)[kElems],
+                                           const uint32_t (&u1)[kElems], const uint32_t (&u2)[kElems],
+                                           const uint32_t (&u3)[kElems], const uint32_t (&ng)[kElems],
+                                           const uint32_t* table, uint8_t* dst, size_t plane_stride) {
+  (planes_one<Is>(u0, u1, u2, u3, ng, table, dst, plane_stride), ...);
+}
+
+// MODE 0: magnitude plane (1 plane); MODE 1: residue digit planes for the
+// first R moduli (R is a template parameter so the modulus loop unrolls and
+// every per-modulus constant and plane offset is known at compile time).
+template <int MODE, int R>
+__global__ void __launch_bounds__(kDecThreads) planes_kernel(OperandView X0, OperandView X1, int blocks0, int64_t k,
+                                                             int64_t k_pad, int clamp_c, int rn,
+                                                             const __grid_constant__ Oz2Moduli mods) {
   extern __shared__ uint32_t table[];
+  const bool second = static_cast<int>(blockIdx.x) >= blocks0;
+  const OperandView X = second ? X1 : X0;
+  const int bid = second ? blockIdx.x - blocks0 : blockIdx.x;
+  const int nblocks = second ? gridDim.x - blocks0 : blocks0;
   if (MODE == 1) {
-    for (int t = threadIdx.x; t < mods.table_entries; t += blockDim.x) table[t] = table_g[t];
+    for (int t = threadIdx.x; t < mods.table_entries; t += blockDim.x) table[t] = X.table[t];
     __syncthreads();
   }
   const int64_t row_tiles = (X.rows + kRowsPerBlock - 1) / kRowsPerBlock;
-  const int64_t k_tiles = k_pad / (2 * kElems);
-  const int64_t ntiles = row_tiles * k_tiles;
-  const int half = threadIdx.x & 1;
-  const int rloc = threadIdx.x >> 1;
+  const int64_t ntiles = row_tiles * (k_pad / kSeg);
+  const int quarter = threadIdx.x & (kQuad - 1);
+  const int rloc = threadIdx.x / kQuad;
   const size_t plane_stride = static_cast<size_t>(X.rows) * k_pad;
 
-  for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+  for (int64_t tile = bid; tile < ntiles; tile += nblocks) {
     const int64_t kt = tile / row_tiles;  // consecutive blocks share a k-slice of many rows
-    const int64_t rt = tile - kt * row_tiles;
-    const int64_t row = rt * kRowsPerBlock + rloc;
+    const int64_t row = (tile - kt * row_tiles) * kRowsPerBlock + rloc;
     if (row >= X.rows) continue;
-    const int64_t l0 = kt * (2 * kElems) + half * kElems;
-    const uint8_t flag = X.flag[row];
+    const int64_t l0 = kt * kSeg + quarter * kElems;
+    double x[kElems];
+    load8(X, row, l0, k, x);  // entries of rows zeroed by the flags are replaced below
+    const bool zero_row = (X.flag[row] & 2) != 0;
     const int ex = X.exps[row];
-    const bool zero_row = (flag & 2) != 0;
     uint8_t* dst = X.out + static_cast<size_t>(row) * k_pad + l0;
+    if (zero_row) {
+#pragma unroll
+      for (int e = 0; e < kElems; ++e) x[e] = 0.0;
+    }
 
     if (MODE == 0) {
       uint32_t code[kElems];
 #pragma unroll
       for (int e = 0; e < kElems; ++e) {
-        int64_t l = l0 + e;
-        code[e] = 0;
-        if (!zero_row && l < k) {
-          Split s = split_double(__ldg(X.base + row * X.row_stride + l * X.k_stride));
-          if (s.M) code[e] = e4m3_pow2(max(-clamp_c, ceil_log2_abs(s) - ex));
-        }
+        const Split sp = split_double(x[e]);
+        code[e] = sp.M ? e4m3_pow2(max(-clamp_c, ceil_log2_abs(sp) - ex)) : 0u;
       }
-      uint4 v;
-      v.x = code[0] | (code[1] << 8) | (code[2] << 16) | (code[3] << 24);
-      v.y = code[4] | (code[5] << 8) | (code[6] << 16) | (code[7] << 24);
-      v.z = code[8] | (code[9] << 8) | (code[10] << 16) | (code[11] << 24);
-      v.w = code[12] | (code[13] << 8) | (code[14] << 16) | (code[15] << 24);
-      *reinterpret_cast<uint4*>(dst) = v;
+      *reinterpret_cast<uint2*>(dst) = make_uint2(code[0] | (code[1] << 8) | (code[2] << 16) | (code[3] << 24),
+                                                  code[4] | (code[5] << 8) | (code[6] << 16) | (code[7] << 24));
     } else {
-      // Quantise (Eq. scale) and split |Ã| into 16-bit limbs.
-      uint32_t lo[kElems], hi[kElems];
-      uint32_t negmask = 0;
+      // Quantise (Eq. scale) and split Ã, as a 64-bit two's complement word,
+      // into 16-bit limbs; the sign enters the residue as one more term,
+      // neg·((-2^64) mod m).
+      uint32_t u0[kElems], u1[kElems], u2[kElems], u3[kElems], ng[kElems];
 #pragma unroll
       for (int e = 0; e < kElems; ++e) {
-        int64_t l = l0 + e;
-        unsigned long long a = 0;
-        if (!zero_row && l < k) {
-          Split s = split_double(__ldg(X.base + row * X.row_stride + l * X.k_stride));
-          a = quantise_abs(s, ex, rn != 0);
-          if (s.neg && a) negmask |= 1u << e;
-        }
-        lo[e] = static_cast<uint32_t>(a);
-        hi[e] = static_cast<uint32_t>(a >> 32);
+        const Split sp = split_double(x[e]);
+        const unsigned long long a = quantise_abs(sp, ex, rn != 0);
+        const bool neg = sp.neg && a != 0;
+        const unsigned long long t = neg ? 0ull - a : a;
+        const uint32_t lo = static_cast<uint32_t>(t), hi = static_cast<uint32_t>(t >> 32);
+        u0[e] = lo & 0xFFFFu;
+        u1[e] = lo >> 16;
+        u2[e] = hi & 0xFFFFu;
+        u3[e] = hi >> 16;
+        ng[e] = neg ? 1u : 0u;
       }
-#pragma unroll 1
-      for (int i = 0; i < mods.r; ++i) {
-        const uint32_t mi = static_cast<uint32_t>(mods.m[i]);
-        const uint32_t mg = mods.magic[i];
-        const int sh = mods.magic_sh[i];
-        const uint32_t c1 = mods.limb[i][1], c2 = mods.limb[i][2], c3 = mods.limb[i][3];
-        const uint32_t noff = static_cast<uint32_t>(mods.negoff[i]);
-        const uint32_t* tab = table + mods.table_off[i];
-        uint32_t w[kElems];
-#pragma unroll
-        for (int e = 0; e < kElems; ++e) {
-          // |Ã| mod m from the limbs: y = u0 + u1·(2^16 mod m) + u2·(2^32 mod m) + u3·(2^48 mod m)
-          uint32_t y = (lo[e] & 0xFFFFu) + (lo[e] >> 16) * c1 + (hi[e] & 0xFFFFu) * c2 +
-                       (hi[e] >> 16) * c3;
-          y = ((negmask >> e) & 1u) ? noff - y : y;  // residue of -|Ã|
-          uint32_t r = mod_magic(y, mi, mg, sh);
-          w[e] = tab[r];                              // packed E4M3 planes of centred(r)
-        }
-        const int np = mods.sq_base[i] ? 2 : 3;
-        uint8_t* pdst = dst + static_cast<size_t>(mods.plane_off[i]) * plane_stride;
-        for (int p = 0; p < np; ++p) {
-          uint4 v;
-          v.x = gather_byte(w[0], w[1], w[2], w[3], p);
-          v.y = gather_byte(w[4], w[5], w[6], w[7], p);
-          v.z = gather_byte(w[8], w[9], w[10], w[11], p);
-          v.w = gather_byte(w[12], w[13], w[14], w[15], p);
-          *reinterpret_cast<uint4*>(pdst + p * plane_stride) = v;
-        }
-      }
+      planes_all(std::make_integer_sequence<int, R>{}, u0, u1, u2, u3, ng, table, dst, plane_stride);
     }
   }
 }
 
-static int grid_for(int64_t rows, int64_t k_pad) {
-  int64_t tiles = ((rows + kRowsPerBlock - 1) / kRowsPerBlock) * (k_pad / (2 * kElems));
+static int num_sms() {
   int dev = 0, sms = 148;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  int64_t cap = static_cast<int64_t>(sms) * 8;
-  return static_cast<int>(tiles < cap ? (tiles > 0 ? tiles : 1) : cap);
+  return sms;
+}
+
+static int64_t tiles_of(int64_t rows, int64_t k_pad) {
+  return ((rows + kRowsPerBlock - 1) / kRowsPerBlock) * (k_pad / kSeg);
+}
+
+// Split a grid of about `blocks_per_sm` × SMs blocks between the two operands
+// in proportion to their tiles.
+static void split_grid(int64_t t0, int64_t t1, int blocks_per_sm, int* g0, int* g1) {
+  const int64_t cap = static_cast<int64_t>(num_sms()) * blocks_per_sm;
+  const int64_t tot = t0 + t1;
+  int64_t b0 = t0 ? std::max<int64_t>(1, std::min<int64_t>(t0, cap * t0 / std::max<int64_t>(tot, 1))) : 0;
+  int64_t b1 = t1 ? std::max<int64_t>(1, std::min<int64_t>(t1, cap - b0)) : 0;
+  *g0 = static_cast<int>(b0);
+  *g1 = static_cast<int>(b1);
+}
+
+static int vec_ok(const double* base, int64_t row_stride, int64_t k_stride) {
+  return k_stride == 1 && (row_stride % 2 == 0) && (reinterpret_cast<uintptr_t>(base) % 16 == 0);
 }
 
 cudaError_t launch_magnitude_planes(int64_t m, int64_t n, int64_t k, const double* A,
@@ -202,16 +247,14 @@ cudaError_t launch_magnitude_planes(int64_t m, int64_t n, int64_t k, const doubl
   int c = (24 - lk) / 2;
   c = c < 0 ? 0 : (c > kMagClampMax ? kMagClampMax : c);
   Oz2Moduli dummy{};
-  if (m > 0) {
-    OperandView va{A, 1, lda, m, ra, row_flag, mag_a};
-    count_launch();
-    planes_kernel<0><<<grid_for(m, k_pad), kDecThreads, 0, st>>>(va, k, k_pad, c, 0, dummy, nullptr);
-  }
-  if (n > 0) {
-    OperandView vb{B, ldb, 1, n, cb, col_flag, mag_b};
-    count_launch();
-    planes_kernel<0><<<grid_for(n, k_pad), kDecThreads, 0, st>>>(vb, k, k_pad, c, 0, dummy, nullptr);
-  }
+  OperandView va{A, 1, lda, m, ra, row_flag, mag_a, nullptr, 0};
+  OperandView vb{B, ldb, 1, n, cb, col_flag, mag_b, nullptr, vec_ok(B, ldb, 1)};
+  int g0, g1;
+  split_grid(m ? tiles_of(m, k_pad) : 0, n ? tiles_of(n, k_pad) : 0, 8, &g0, &g1);
+  if (g0 + g1 == 0) return cudaSuccess;
+  if (g0 == 0) va = vb;
+  count_launch();
+  planes_kernel<0, 0><<<g0 + g1, kDecThreads, 0, st>>>(va, vb, g0, k, k_pad, c, 0, dummy);
   return cudaGetLastError();
 }
 
@@ -221,21 +264,32 @@ cudaError_t launch_deconstruct(int64_t m, int64_t n, int64_t k, const Oz2Moduli&
                                const uint8_t* row_flag, const uint8_t* col_flag, int quant,
                                uint8_t* planes_a, uint8_t* planes_b, cudaStream_t st) {
   const int64_t k_pad = (k + kKPad - 1) / kKPad * kKPad;
-  size_t smem = sizeof(uint32_t) * mods.table_entries;
-  cudaError_t err = cudaFuncSetAttribute(planes_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
-  if (err != cudaSuccess) return err;
+  const size_t smem = sizeof(uint32_t) * mods.table_entries;
   const int rn = quant == OZ2_QUANT_RN;
-  if (m > 0) {
-    OperandView va{A, 1, lda, m, d, row_flag, planes_a};
-    count_launch();
-    planes_kernel<1><<<grid_for(m, k_pad), kDecThreads, smem, st>>>(va, k, k_pad, 0, rn, mods, table_a);
+  OperandView va{A, 1, lda, m, d, row_flag, planes_a, table_a, 0};
+  OperandView vb{B, ldb, 1, n, e, col_flag, planes_b, table_b, vec_ok(B, ldb, 1)};
+  int g0, g1;
+  split_grid(m ? tiles_of(m, k_pad) : 0, n ? tiles_of(n, k_pad) : 0, 4, &g0, &g1);
+  if (g0 + g1 == 0) return cudaSuccess;
+  if (g0 == 0) va = vb;
+  cudaError_t err = cudaSuccess;
+  count_launch();
+  switch (mods.r) {
+#define OZ2_DEC_CASE(R)                                                                                     \
+  case R:                                                                                                   \
+    err = cudaFuncSetAttribute(planes_kernel<1, R>, cudaFuncAttributeMaxDynamicSharedMemorySize,            \
+                               static_cast<int>(smem));                                                     \
+    if (err == cudaSuccess)                                                                                 \
+      planes_kernel<1, R><<<g0 + g1, kDecThreads, smem, st>>>(va, vb, g0, k, k_pad, 0, rn, mods);          \
+    break;
+    OZ2_DEC_CASE(1) OZ2_DEC_CASE(2) OZ2_DEC_CASE(3) OZ2_DEC_CASE(4) OZ2_DEC_CASE(5) OZ2_DEC_CASE(6)
+    OZ2_DEC_CASE(7) OZ2_DEC_CASE(8) OZ2_DEC_CASE(9) OZ2_DEC_CASE(10) OZ2_DEC_CASE(11) OZ2_DEC_CASE(12)
+    OZ2_DEC_CASE(13) OZ2_DEC_CASE(14) OZ2_DEC_CASE(15) OZ2_DEC_CASE(16)
+#undef OZ2_DEC_CASE
+    default:
+      return cudaErrorInvalidValue;
   }
-  if (n > 0) {
-    OperandView vb{B, ldb, 1, n, e, col_flag, planes_b};
-    count_launch();
-    planes_kernel<1><<<grid_for(n, k_pad), kDecThreads, smem, st>>>(vb, k, k_pad, 0, rn, mods, table_b);
-  }
+  if (err != cudaSuccess) return err;
   return cudaGetLastError();
 }
 

@@ -42,9 +42,10 @@ __global__ void scan_a_kernel(int64_t m, int64_t k, const double* __restrict__ A
   if (best) atomicMax(key + i, best);
 }
 
-// Columns of column-major B: warp per column, lanes over l, grid.y splits k.
+// Columns of column-major B: warp per column, lanes over l, grid.y splits k
+// into even-sized chunks; 16-byte loads when the column start is aligned.
 __global__ void scan_b_kernel(int64_t n, int64_t k, const double* __restrict__ B, int64_t ldb,
-                              int chunk, int* __restrict__ key) {
+                              int chunk, int vec, int* __restrict__ key) {
   int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   int64_t j = blockIdx.x * (int64_t)(blockDim.x >> 5) + warp;
   if (j >= n) return;
@@ -52,11 +53,27 @@ __global__ void scan_b_kernel(int64_t n, int64_t k, const double* __restrict__ B
   int64_t l1 = min(k, l0 + chunk);
   const double* col = B + j * ldb;
   int best = 0;
-  int64_t l = l0 + lane;
-  for (; l + 96 < l1; l += 128)
-    best = max(best, max(max(scan_key(__ldg(col + l)), scan_key(__ldg(col + l + 32))),
-                         max(scan_key(__ldg(col + l + 64)), scan_key(__ldg(col + l + 96)))));
-  for (; l < l1; l += 32) best = max(best, scan_key(__ldg(col + l)));
+  if (vec) {
+    const double2* c2 = reinterpret_cast<const double2*>(col);
+    const int64_t p1 = l1 >> 1;  // pairs fully inside [l0, l1) (l0 is even)
+    int64_t p = (l0 >> 1) + lane;
+    for (; p + 96 < p1; p += 128) {
+      const double2 a = __ldg(c2 + p), b = __ldg(c2 + p + 32), c = __ldg(c2 + p + 64), d = __ldg(c2 + p + 96);
+      best = max(best, max(max(max(scan_key(a.x), scan_key(a.y)), max(scan_key(b.x), scan_key(b.y))),
+                           max(max(scan_key(c.x), scan_key(c.y)), max(scan_key(d.x), scan_key(d.y)))));
+    }
+    for (; p < p1; p += 32) {
+      const double2 a = __ldg(c2 + p);
+      best = max(best, max(scan_key(a.x), scan_key(a.y)));
+    }
+    if ((l1 & 1) && lane == 0) best = max(best, scan_key(__ldg(col + l1 - 1)));
+  } else {
+    int64_t l = l0 + lane;
+    for (; l + 96 < l1; l += 128)
+      best = max(best, max(max(scan_key(__ldg(col + l)), scan_key(__ldg(col + l + 32))),
+                           max(scan_key(__ldg(col + l + 64)), scan_key(__ldg(col + l + 96)))));
+    for (; l < l1; l += 32) best = max(best, scan_key(__ldg(col + l)));
+  }
   best = __reduce_max_sync(0xffffffffu, best);
   if (lane == 0 && best) atomicMax(key + j, best);
 }
@@ -133,7 +150,7 @@ cudaError_t launch_scan(int64_t m, int64_t n, int64_t k, const double* A, int64_
   if (m > 0 && (err = cudaMemsetAsync(out.ra, 0, sizeof(int) * m, st)) != cudaSuccess) return err;
   if (n > 0 && (err = cudaMemsetAsync(out.cb, 0, sizeof(int) * n, st)) != cudaSuccess) return err;
   if (k > 0) {
-    int chunk = 256;
+    int chunk = 64;
     int64_t ks = (k + chunk - 1) / chunk;
     if (ks > 65535) {
       chunk = static_cast<int>((k + 65534) / 65535);
@@ -144,16 +161,17 @@ cudaError_t launch_scan(int64_t m, int64_t n, int64_t k, const double* A, int64_
       count_launch();
       scan_a_kernel<<<g, 256, 0, st>>>(m, k, A, lda, chunk, out.ra);
     }
-    int bchunk = 4096;
+    int bchunk = 1024;
     int64_t bks = (k + bchunk - 1) / bchunk;
     if (bks > 65535) {
-      bchunk = static_cast<int>((k + 65534) / 65535);
+      bchunk = static_cast<int>((k + 65534) / 65535 + 1) & ~1;
       bks = (k + bchunk - 1) / bchunk;
     }
     if (n > 0) {
+      const int vec = (ldb % 2 == 0) && (reinterpret_cast<uintptr_t>(B) % 16 == 0);
       dim3 g(static_cast<unsigned>((n + 7) / 8), static_cast<unsigned>(bks));
       count_launch();
-      scan_b_kernel<<<g, 256, 0, st>>>(n, k, B, ldb, bchunk, out.cb);
+      scan_b_kernel<<<g, 256, 0, st>>>(n, k, B, ldb, bchunk, vec, out.cb);
     }
   }
   count_launch();

@@ -153,6 +153,32 @@ static Oz2Moduli build_moduli(int r, int quant) {
   }
   c.nplanes = plane;
   c.table_entries = toff;
+  // Direct-CRT constants.
+  for (int k = 0; k < r; ++k) {
+    const int mk = kModuliAll[k];
+    uint32_t W[6] = {1, 0, 0, 0, 0, 0};  // Π_{j≠k} m_j, then × y_k
+    long long pm = 1;                    // Π_{j≠k} m_j mod m_k
+    for (int j = 0; j < r; ++j) {
+      if (j == k) continue;
+      u64 carry = 0;
+      for (int t = 0; t < 6; ++t) {
+        const u64 v = static_cast<u64>(W[t]) * static_cast<u64>(kModuliAll[j]) + carry;
+        W[t] = static_cast<uint32_t>(v);
+        carry = v >> 32;
+      }
+      pm = (pm * kModuliAll[j]) % mk;
+    }
+    const int y = mod_inverse(pm, mk);
+    u64 carry = 0;
+    for (int t = 0; t < 6; ++t) {
+      const u64 v = static_cast<u64>(W[t]) * static_cast<u64>(y) + carry;
+      W[t] = static_cast<uint32_t>(v);
+      carry = v >> 32;
+    }
+    for (int t = 0; t < 5; ++t) c.crtw[k][t] = W[t];
+    c.crtf[k] = static_cast<uint32_t>(((static_cast<u64>(y) << 32) + static_cast<u64>(mk / 2)) / static_cast<u64>(mk));
+    c.coff[k] = mk * ((32768 + mk - 1) / mk);
+  }
   u64 M[3] = {1, 0, 0};
   for (int i = 0; i < r; ++i) mul3(M, static_cast<u64>(kModuliAll[i]));
   for (int i = 0; i < 3; ++i) c.M[i] = M[i];

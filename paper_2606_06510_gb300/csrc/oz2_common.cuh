@@ -25,6 +25,59 @@ constexpr int kFallbackWindow = 128;   // binades from the median (fallback)
 constexpr int kKSlabSquare = 32768;
 constexpr int kKSlabMerged = 4096;
 
+// The modulus list (§2.5: the published set S in the order the paper lists
+// it, then the extension primes for r = 13..16) and per-modulus constants
+// derived from it at compile time.
+constexpr int kModuliList[kMaxModuli] = {1089, 1024, 961, 841, 625, 529, 511, 509,
+                                         503,  499,  491, 487, 479, 467, 463, 461};
+
+struct ModConst {
+  int m;
+  int s;          // square base, 0 for nonsquare moduli
+  int plane_off;  // first plane of this modulus
+  int table_off;  // first entry of this modulus in the digit-plane table
+  uint32_t limb1, limb2, limb3;  // 2^16, 2^32, 2^48 mod m
+  uint32_t neg64;                // (-2^64) mod m
+  uint32_t magic;                // ⌈2^(32+sh)/m⌉
+  int sh;                        // ⌊log2(m-1)⌋
+};
+
+constexpr int ce_isqrt(int m) {
+  int s = 0;
+  while ((s + 1) * (s + 1) <= m) ++s;
+  return s * s == m ? s : 0;
+}
+constexpr int ce_log2_floor(unsigned v) {
+  int r = -1;
+  while (v) {
+    v >>= 1;
+    ++r;
+  }
+  return r;
+}
+constexpr ModConst mod_const(int i) {
+  ModConst c{};
+  int plane = 0, toff = 0;
+  for (int j = 0; j < i; ++j) {
+    plane += ce_isqrt(kModuliList[j]) ? 2 : 3;
+    toff += kModuliList[j];
+  }
+  const int m = kModuliList[i];
+  c.m = m;
+  c.s = ce_isqrt(m);
+  c.plane_off = plane;
+  c.table_off = toff;
+  const unsigned long long um = static_cast<unsigned long long>(m);
+  c.limb1 = static_cast<uint32_t>((1ull << 16) % um);
+  c.limb2 = static_cast<uint32_t>((1ull << 32) % um);
+  c.limb3 = static_cast<uint32_t>((1ull << 48) % um);
+  const unsigned long long two64 = ((~0ull) % um + 1) % um;  // 2^64 mod m
+  c.neg64 = static_cast<uint32_t>((um - two64) % um);
+  c.sh = ce_log2_floor(static_cast<unsigned>(m - 1));
+  c.magic = static_cast<uint32_t>(((1ull << (32 + c.sh)) + um - 1) / um);
+  return c;
+}
+
 // Device status word values (stored in Oz2Device::status).
 constexpr int kStatusTimeout = 1;
 
@@ -49,6 +102,12 @@ struct Oz2Moduli {
   // M and ⌈M/2⌉ as 3×64-bit little-endian limbs.
   unsigned long long M[3];
   unsigned long long Mhalf[3];
+  // Direct CRT (fast path of the reconstruction): W_k = (M/m_k)·y_k with
+  // y_k = (M/m_k)^-1 mod m_k as 32-bit limbs, F_k = round(2^32·y_k/m_k), and
+  // coff_k = m_k·⌈2^15/m_k⌉ (makes any int16 residue nonnegative).
+  uint32_t crtw[kMaxModuli][5];
+  uint32_t crtf[kMaxModuli];
+  int coff[kMaxModuli];
   int table_entries;            // Σ m_i
 };
 

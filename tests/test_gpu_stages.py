@@ -206,6 +206,36 @@ def test_reconstruct(oz):
                 assert C[i, j] == want and np.signbit(C[i, j]) == np.signbit(want), (r, i, j)
 
 
+def test_reconstruct_near_the_range_boundary(oz):
+    """Integers at and next to ±M/2, where the fast reconstruction defers to
+    Garner's algorithm, and a band of values around them."""
+    import random
+    import torch
+    for r in (3, 12, 13, 16):
+        mods = orc.moduli(r)
+        M = orc.modulus_product(mods)
+        lo, hi = -(M // 2), M - M // 2 - 1
+        rng = random.Random(r)
+        xs = [lo, lo + 1, hi, hi - 1, 0, 1, -1]
+        band = max(1, M >> 13)
+        xs += [lo + rng.randrange(band) for _ in range(60)] + [hi - rng.randrange(band) for _ in range(60)]
+        xs += [rng.randrange(lo, hi + 1) for _ in range(60)]
+        m, n = len(xs), 3
+        R = np.zeros((r, m, n), dtype=np.int64)
+        for i, x in enumerate(xs):
+            for k, mk in enumerate(mods):
+                R[k, i, :] = int(orc.centred(x % mk, mk))
+        d = np.full(m, 5, dtype=np.int64)
+        e = np.array([0, 40, -1100], dtype=np.int64)
+        res = torch.from_numpy(R.astype(np.int16)).cuda()
+        C = oz.oz2_reconstruct(res, torch.from_numpy(d.astype(np.int32)).cuda(),
+                               torch.from_numpy(e.astype(np.int32)).cuda(), m, n, r).cpu().numpy()
+        for i, x in enumerate(xs):
+            for j in range(n):
+                want = orc.unscale_one(x, -int(d[i]) - int(e[j]))
+                assert C[i, j] == want and np.signbit(C[i, j]) == np.signbit(want), (r, i, j)
+
+
 def test_fallback_rows_and_columns(oz):
     import torch
     m, n, k = 70, 60, 50
