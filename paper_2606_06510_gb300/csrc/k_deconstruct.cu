@@ -2,12 +2,16 @@
 // and the magnitude planes of the "+1" pass (§2.4).
 //
 // One thread handles 8 consecutive k-entries of one row of the operand (a row
-// of A, or a column of B seen as a row of Bᵀ); the four threads of a lane
-// quad cover 32 consecutive k-entries, so every plane row segment they write
-// is one full 32-byte sector (8-byte stores per thread).  A is column-major:
-// a warp's 8 row-quads read 8 consecutive rows of 4 columns per load.  B's
-// rows are contiguous in k and are read with 16-byte vector loads.  One
-// launch covers both operands: the first blocks work on A, the rest on B.
+// of A, or a column of B seen as a row of Bᵀ).  In the deconstruction, 16
+// threads share a row and cover 128 consecutive k-entries, so each plane row
+// segment they write is one full 128-byte line (8-byte stores per thread);
+// partial lines written by different blocks at different times cost the
+// memory system a read-modify-write each.  The magnitude pass writes one
+// plane only and is faster with 4 threads per row (32-byte segments, more
+// rows in flight per block).  A is column-major: the threads of a warp that
+// load the same k-entries read consecutive rows.  B's rows are contiguous in
+// k and are read with 16-byte vector loads.  One launch covers both
+// operands: the first blocks work on A, the rest on B.
 #include <algorithm>
 #include <utility>
 
@@ -15,11 +19,18 @@
 
 namespace oz2 {
 
-constexpr int kElems = 8;                // k-entries per thread
-constexpr int kQuad = 4;                 // threads per 32-entry row segment
-constexpr int kSeg = kElems * kQuad;     // k-entries per tile column
+constexpr int kElems = 8;  // k-entries per thread
 constexpr int kDecThreads = 256;
-constexpr int kRowsPerBlock = kDecThreads / kQuad;  // 64
+
+// Tile shape of each pass: threads per row, k-entries per tile column (a
+// divisor of the k padding) and rows per block.
+template <int MODE>
+struct TileShape {
+  static constexpr int kThreadsPerRow = MODE == 0 ? 4 : 16;
+  static constexpr int kSeg = kElems * kThreadsPerRow;
+  static constexpr int kRows = kDecThreads / kThreadsPerRow;
+};
+static_assert(kKPad % TileShape<0>::kSeg == 0 && kKPad % TileShape<1>::kSeg == 0, "tile column must divide k_pad");
 
 // Integer significand M and exponent x with |x| = M·2^x (M < 2^53), or M = 0.
 struct Split {
@@ -158,17 +169,18 @@ __global__ void __launch_bounds__(kDecThreads) planes_kernel(OperandView X0, Ope
     for (int t = threadIdx.x; t < mods.table_entries; t += blockDim.x) table[t] = X.table[t];
     __syncthreads();
   }
-  const int64_t row_tiles = (X.rows + kRowsPerBlock - 1) / kRowsPerBlock;
-  const int64_t ntiles = row_tiles * (k_pad / kSeg);
-  const int quarter = threadIdx.x & (kQuad - 1);
-  const int rloc = threadIdx.x / kQuad;
+  using TS = TileShape<MODE>;
+  const int64_t row_tiles = (X.rows + TS::kRows - 1) / TS::kRows;
+  const int64_t ntiles = row_tiles * (k_pad / TS::kSeg);
+  const int part = threadIdx.x & (TS::kThreadsPerRow - 1);
+  const int rloc = threadIdx.x / TS::kThreadsPerRow;
   const size_t plane_stride = static_cast<size_t>(X.rows) * k_pad;
 
   for (int64_t tile = bid; tile < ntiles; tile += nblocks) {
     const int64_t kt = tile / row_tiles;  // consecutive blocks share a k-slice of many rows
-    const int64_t row = (tile - kt * row_tiles) * kRowsPerBlock + rloc;
+    const int64_t row = (tile - kt * row_tiles) * TS::kRows + rloc;
     if (row >= X.rows) continue;
-    const int64_t l0 = kt * kSeg + quarter * kElems;
+    const int64_t l0 = kt * TS::kSeg + part * kElems;
     double x[kElems];
     load8(X, row, l0, k, x);  // entries of rows zeroed by the flags are replaced below
     const bool zero_row = (X.flag[row] & 2) != 0;
@@ -218,8 +230,10 @@ static int num_sms() {
   return sms;
 }
 
+template <int MODE>
 static int64_t tiles_of(int64_t rows, int64_t k_pad) {
-  return ((rows + kRowsPerBlock - 1) / kRowsPerBlock) * (k_pad / kSeg);
+  using TS = TileShape<MODE>;
+  return ((rows + TS::kRows - 1) / TS::kRows) * (k_pad / TS::kSeg);
 }
 
 // Split a grid of about `blocks_per_sm` × SMs blocks between the two operands
@@ -250,7 +264,7 @@ cudaError_t launch_magnitude_planes(int64_t m, int64_t n, int64_t k, const doubl
   OperandView va{A, 1, lda, m, ra, row_flag, mag_a, nullptr, 0};
   OperandView vb{B, ldb, 1, n, cb, col_flag, mag_b, nullptr, vec_ok(B, ldb, 1)};
   int g0, g1;
-  split_grid(m ? tiles_of(m, k_pad) : 0, n ? tiles_of(n, k_pad) : 0, 8, &g0, &g1);
+  split_grid(m ? tiles_of<0>(m, k_pad) : 0, n ? tiles_of<0>(n, k_pad) : 0, 8, &g0, &g1);
   if (g0 + g1 == 0) return cudaSuccess;
   if (g0 == 0) va = vb;
   count_launch();
@@ -269,7 +283,7 @@ cudaError_t launch_deconstruct(int64_t m, int64_t n, int64_t k, const Oz2Moduli&
   OperandView va{A, 1, lda, m, d, row_flag, planes_a, table_a, 0};
   OperandView vb{B, ldb, 1, n, e, col_flag, planes_b, table_b, vec_ok(B, ldb, 1)};
   int g0, g1;
-  split_grid(m ? tiles_of(m, k_pad) : 0, n ? tiles_of(n, k_pad) : 0, 4, &g0, &g1);
+  split_grid(m ? tiles_of<1>(m, k_pad) : 0, n ? tiles_of<1>(n, k_pad) : 0, 4, &g0, &g1);
   if (g0 + g1 == 0) return cudaSuccess;
   if (g0 == 0) va = vb;
   cudaError_t err = cudaSuccess;
