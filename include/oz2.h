@@ -154,14 +154,17 @@ int oz2_dgemm_ex(int64_t m, int64_t n, int64_t k,
  *   urow[m]               float  max_j U_ij of the "+1" GEMM (R2)
  *   mag_a, mag_b          uint8  magnitude planes Â (m×k_pad), B̂ (n×k_pad)
  *   planes_a, planes_b    uint8  E4M3 digit planes, see oz2_plane_layout
- *   residues              int16  r matrices C^(i), each m×n row-major
- *                                (ld = n), centred in [-⌊m_i/2⌋, m_i-1-⌊m_i/2⌋]
+ *   residues              int16  r matrices C^(i), each m×n column-major
+ *                                with ld = res_ld (matrix i starts at element
+ *                                i·n·res_ld), centred in
+ *                                [-⌊m_i/2⌋, m_i-1-⌊m_i/2⌋]
  */
 typedef struct {
   size_t ra, cb, row_flag, col_flag, d, e, urow, misc;
   size_t mag_a, mag_b, planes_a, planes_b, residues, total;
   int64_t k_pad;             /* k rounded up to a multiple of 128 */
   int32_t num_planes;        /* stored planes per operand element */
+  int64_t res_ld;            /* m rounded up to a multiple of 8 */
 } oz2_ws_layout;
 int oz2_workspace_layout(int64_t m, int64_t n, int64_t k, int num_moduli,
                          oz2_ws_layout* out);
@@ -228,24 +231,29 @@ int oz2_deconstruct(int64_t m, int64_t n, int64_t k, int num_moduli,
 
 /* Stage 4 (Eq. modgemm, Eq. sq-shortcut, Eq. kar): from digit planes in
  * the oz2_plane_layout order (k_pad = k rounded up to 128), the residue
- * matrices C^(i) = (A^(i) B^(i)) mod m_i, centred, r × (m×n row-major,
- * ld = n) int16.  Three FP8 tcgen05 MMAs per modulus into two FP32
- * accumulators with exact accumulation (Eq. accum-exact), reduced mod m_i
- * every K-slab (32768 for square moduli, 4096 for nonsquare ones). */
+ * matrices C^(i) = (A^(i) B^(i)) mod m_i, centred, as r int16 matrices,
+ * each m×n column-major with leading dimension ldr ≥ m (matrix i starts at
+ * element i·n·ldr; rows m..ldr-1 are not written).  Three FP8 tcgen05 MMAs
+ * per modulus into two FP32 accumulators with exact accumulation (Eq.
+ * accum-exact), reduced mod m_i every K-slab (32768 for square moduli, 4096
+ * for nonsquare ones).  ldr < m → OZ2_ERR_INVALID_ARG. */
 int oz2_residue_gemm(int64_t m, int64_t n, int64_t k, int num_moduli,
                      const uint8_t* d_planes_a, const uint8_t* d_planes_b,
-                     int16_t* d_residues, void* stream);
+                     int16_t* d_residues, int64_t ldr, void* stream);
 
 /* Diagnostic twin of oz2_residue_gemm on CUDA cores (same products, same
- * epilogue arithmetic, sequential k order); slow. */
+ * epilogue arithmetic, sequential k order, same output layout); slow. */
 int oz2_residue_gemm_simt(int64_t m, int64_t n, int64_t k, int num_moduli,
                           const uint8_t* d_planes_a, const uint8_t* d_planes_b,
-                          int16_t* d_residues, void* stream);
+                          int16_t* d_residues, int64_t ldr, void* stream);
 
 /* Stage 5 (Eq. garner, App. A; Algorithm 1 unscale): C_ij = RN_fp64(X_ij ·
  * 2^-(d_i+e_j)) with X_ij ∈ [-M/2, M/2) the integer whose residues are
- * C^(i)_ij.  residues: r × (m×n row-major, ld = ldr ≥ n; matrix i starts
- * at element i·m·ldr) int16, centred or not. */
+ * C^(i)_ij.  residues: r int16 matrices, each m×n column-major with
+ * leading dimension ldr ≥ m (matrix i starts at element i·n·ldr), the
+ * layout oz2_residue_gemm writes; each entry any representative of its class
+ * with |C^(i)_ij| < m_i (oz2_residue_gemm writes the centred one).  Entries
+ * outside that range give unspecified values (never a fault). */
 int oz2_reconstruct(int64_t m, int64_t n, int num_moduli,
                     const int16_t* d_residues, int64_t ldr,
                     const int32_t* d_d, const int32_t* d_e,

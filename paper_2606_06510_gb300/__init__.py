@@ -47,7 +47,7 @@ class oz2_ws_layout(ctypes.Structure):
     _fields_ = [(name, ctypes.c_size_t) for name in
                 ("ra", "cb", "row_flag", "col_flag", "d", "e", "urow", "misc",
                  "mag_a", "mag_b", "planes_a", "planes_b", "residues", "total")] + \
-               [("k_pad", ctypes.c_int64), ("num_planes", ctypes.c_int32)]
+               [("k_pad", ctypes.c_int64), ("num_planes", ctypes.c_int32), ("res_ld", ctypes.c_int64)]
 
 
 _I64, _P, _I, _U, _SZ = ctypes.c_int64, ctypes.c_void_p, ctypes.c_int, ctypes.c_uint, ctypes.c_size_t
@@ -65,8 +65,8 @@ _SIGS = {
     "oz2_scan": (_I, [_I64, _I64, _I64, _P, _I64, _P, _I64, _U, _P, _P, _P, _P, _P]),
     "oz2_scale": (_I, [_I64, _I64, _I64, _I, _P, _I64, _P, _I64, _P, _P, _P, _P, _I, _I, _P, _P, _P, _P, _P, _P]),
     "oz2_deconstruct": (_I, [_I64, _I64, _I64, _I, _P, _I64, _P, _I64, _P, _P, _P, _P, _I, _P, _P, _P]),
-    "oz2_residue_gemm": (_I, [_I64, _I64, _I64, _I, _P, _P, _P, _P]),
-    "oz2_residue_gemm_simt": (_I, [_I64, _I64, _I64, _I, _P, _P, _P, _P]),
+    "oz2_residue_gemm": (_I, [_I64, _I64, _I64, _I, _P, _P, _P, _I64, _P]),
+    "oz2_residue_gemm_simt": (_I, [_I64, _I64, _I64, _I, _P, _P, _P, _I64, _P]),
     "oz2_reconstruct": (_I, [_I64, _I64, _I, _P, _I64, _P, _P, _P, _I64, _P]),
     "oz2_fallback": (_I, [_I64, _I64, _I64, _P, _I64, _P, _I64, _P, _P, _P, _I64, _P]),
     "oz2_native_dgemm": (_I, [_I64, _I64, _I64, _P, _I64, _P, _I64, _P, _I64, _P]),
@@ -259,20 +259,43 @@ def oz2_deconstruct(A, B, d, e, rf, cf, num_moduli=12, quant="tz", stream=None):
     return pa, pb
 
 
+def residue_ld(m: int) -> int:
+    """Leading dimension of the column-major residue matrices (m rounded up to 8)."""
+    return (m + 7) // 8 * 8
+
+
 def oz2_residue_gemm(planes_a, planes_b, m, n, k, num_moduli=12, simt=False, stream=None):
-    """planes: uint8 CUDA tensors (P, rows, k_pad). Returns int16 (r, m, n): r row-major m×n."""
-    res = torch.empty((num_moduli, m, n), dtype=torch.int16, device=planes_a.device)
+    """planes: uint8 CUDA tensors (P, rows, k_pad).  Returns an int16 view of
+    shape (r, m, n) over column-major storage (r, n, ldr), ldr = residue_ld(m)."""
+    ldr = residue_ld(m)
+    res = torch.empty((num_moduli, n, ldr), dtype=torch.int16, device=planes_a.device)
     fn = lib().oz2_residue_gemm_simt if simt else lib().oz2_residue_gemm
-    _check(fn(m, n, k, num_moduli, _ptr(planes_a), _ptr(planes_b), _ptr(res), _stream(stream)),
+    _check(fn(m, n, k, num_moduli, _ptr(planes_a), _ptr(planes_b), _ptr(res), ldr, _stream(stream)),
            "oz2_residue_gemm")
-    return res
+    return res[:, :, :m].transpose(1, 2)
+
+
+def _residue_storage(residues, m, n):
+    """(tensor, ldr) of column-major residue storage for a (r, m, n) tensor:
+    the tensor's own storage when it already has that layout (as the views
+    oz2_residue_gemm returns do), else a column-major copy."""
+    r = residues.shape[0]
+    st = residues.stride()
+    if residues.shape[1:] == (m, n) and st[1] == 1 and st[2] >= max(1, m) and st[0] == n * st[2]:
+        return residues, st[2]
+    ldr = residue_ld(m)
+    buf = torch.zeros((r, n, ldr), dtype=torch.int16, device=residues.device)
+    buf[:, :, :m].copy_(residues.transpose(1, 2))
+    return buf, ldr
 
 
 def oz2_reconstruct(residues, d, e, m, n, num_moduli=12, C=None, stream=None):
-    """residues: int16 CUDA tensor (r, m, n) (row-major m×n per modulus)."""
+    """residues: int16 CUDA tensor (r, m, n); column-major storage per modulus
+    is used as is, any other layout is copied into it first."""
     if C is None:
         C = torch.empty((n, m), dtype=torch.float64, device=residues.device).t()
-    _check(lib().oz2_reconstruct(m, n, num_moduli, _ptr(residues), n, _ptr(d), _ptr(e), _ptr(C), _ld(C),
+    res, ldr = _residue_storage(residues, m, n)
+    _check(lib().oz2_reconstruct(m, n, num_moduli, _ptr(res), ldr, _ptr(d), _ptr(e), _ptr(C), _ld(C),
                                  _stream(stream)), "oz2_reconstruct")
     return C
 
@@ -313,5 +336,6 @@ def workspace_views(ws: torch.Tensor, m: int, n: int, k: int, num_moduli: int) -
         "mag_b": view(L["mag_b"], n * k_pad, torch.uint8, (n, k_pad)),
         "planes_a": view(L["planes_a"], P * m * k_pad, torch.uint8, (P, m, k_pad)),
         "planes_b": view(L["planes_b"], P * n * k_pad, torch.uint8, (P, n, k_pad)),
-        "residues": view(L["residues"], num_moduli * m * n, torch.int16, (num_moduli, m, n)),
+        "residues": view(L["residues"], num_moduli * n * L["res_ld"], torch.int16,
+                         (num_moduli, n, L["res_ld"]))[:, :, :m].transpose(1, 2),
     }

@@ -1,19 +1,22 @@
 // Phase 3 of Ozaki Scheme II (§2.3 Eq. garner, Appendix A; Algorithm 1
-// "C ← D^-1 C̃ E^-1"): Garner mixed-radix digits per output, the integer
-// X = Σ v_k P_{k-1} mapped to [-M/2, M/2), and one correctly rounded
-// (round-to-nearest-even) conversion of X·2^-(d_i+e_j) to FP64, including
-// the subnormal range.
+// "C ← D^-1 C̃ E^-1"): the integer X ∈ [-M/2, M/2) with the given residues
+// and one correctly rounded (round-to-nearest-even) conversion of
+// X·2^-(d_i+e_j) to FP64, including the subnormal range.
 //
-// The reconstruction is computed by the direct CRT sum with a fixed-point
-// quotient (multiply-adds only); Garner's algorithm, the paper's method,
-// takes over in the rare case where that quotient is ambiguous, so every
-// output equals the Garner result exactly.
+// X is computed by the direct CRT sum in fixed point (multiply-adds only);
+// Garner's algorithm, the paper's method, takes over in the rare case where
+// the fixed-point quotient is ambiguous, so every output equals the Garner
+// result exactly.
 //
-// Residues arrive row-major (r matrices of m×n, ld = ldr ≥ n) from the
-// residue GEMM; C is column-major.  A block computes a 32-row × 128-column
-// tile: each thread reads four consecutive residues of one row per modulus
-// (8-byte loads along n), computes its outputs, and the tile is transposed
-// through shared memory so that C is written in 256-byte column segments.
+// Residues arrive column-major (r matrices of m×n, ld = ldr ≥ m) from the
+// residue GEMM and C is column-major, so a thread takes two consecutive
+// rows of a column: one 4-byte load per modulus (a warp reads 128 bytes per
+// modulus) and one 16-byte store of its two results (a warp writes 512
+// contiguous bytes), with no transposition.  Each thread walks a strided
+// set of columns and loads the next column's residues while it computes the
+// current one.  An output that needs Garner's algorithm is marked with a
+// NaN sentinel and recomputed after the loop, which keeps Garner's register
+// footprint out of the loop.
 #include "oz2_common.cuh"
 
 namespace oz2 {
@@ -21,7 +24,6 @@ namespace oz2 {
 typedef unsigned long long u64;
 typedef unsigned __int128 u128;
 
-constexpr int kCrtRows = 32, kCrtCols = 128, kCrtThreads = 256;
 
 // X (L little-endian 32-bit limbs) = X·m + v.  Only the low `nl` limbs can be
 // nonzero afterwards; each limb step is one 32×32+64-bit multiply-add.
@@ -221,92 +223,212 @@ __device__ __forceinline__ bool crt_value_fast(const int (&c)[R], int E, const O
   return true;
 }
 
+// c·(hi·2^32 + lo) mod 2^64 split as a 64-bit part and a 32-bit high-word
+// part: one signed 32×32→64 multiply-add and one 32-bit multiply-add.
+__device__ __forceinline__ void mad_word(int c, int lo, int hi, long long& acc64, uint32_t& acc_hi) {
+  acc64 += static_cast<long long>(c) * lo;
+  acc_hi += static_cast<uint32_t>(c) * static_cast<uint32_t>(hi);
+}
+
+// Nearest double to (-1)^neg·(hi·2^64 + lo)·2^E for hi ≠ 0 (general path).
+__device__ __forceinline__ double round_to_double_big(u64 hi, u64 lo, int E, bool neg) {
+  const int sh = 64 - __clzll(static_cast<long long>(hi));
+  const u64 top = (hi << (64 - sh)) | (lo >> sh);
+  return round_to_double(top, (lo << (64 - sh)) != 0, E + sh, neg);
+}
+
+// Nearest double to X·2^E for X = Hs·2^64 + L (two's complement, |X| < 2^111).
+// The common case (|X| ≥ 2^64, normal result) takes the leading 64 bits with
+// two funnel shifts and lets the hardware conversion round them: a sticky
+// bit for the rest is folded into bit 0, below the rounding position (bit
+// 10), so the conversion's round-to-nearest-even decides as the exact value
+// would.  The exponent is then added to the double's bit pattern.
+__device__ __forceinline__ double finish_words(long long Hs, u64 L, int E) {
+  const bool neg = Hs < 0;
+  u64 hi = static_cast<u64>(Hs), lo = L;
+  if (neg) {
+    lo = 0ull - L;
+    hi = ~hi + (L == 0 ? 1ull : 0ull);
+  }
+  if (hi == 0) return round_to_double(lo, false, E, neg);
+  const uint32_t w3 = static_cast<uint32_t>(hi >> 32), w2 = static_cast<uint32_t>(hi);
+  const uint32_t w1 = static_cast<uint32_t>(lo >> 32), w0 = static_cast<uint32_t>(lo);
+  const int s = w3 ? __clz(w3) : 32 + __clz(w2);  // leading zeros of hi, 17..63
+  const int e2 = E + 127 - s;                      // exponent of the leading bit of X·2^E
+  if (e2 < -1022 || e2 > 1022) return round_to_double_big(hi, lo, E, neg);
+  const bool ge = s >= 32;
+  const uint32_t x3 = ge ? w2 : w3, x2 = ge ? w1 : w2, x1 = ge ? w0 : w1, x0 = ge ? 0u : w0;
+  const int sp = s & 31;
+  const uint32_t th = __funnelshift_l(x2, x3, sp), tl = __funnelshift_l(x1, x2, sp);
+  const bool sticky = ((x1 << sp) | x0) != 0;
+  const u64 top = (static_cast<u64>(th) << 32) | tl | (sticky ? 1ull : 0ull);  // bit 63 set
+  const long long bits = __double_as_longlong(__ull2double_rn(top)) + (static_cast<long long>(E + 64 - s) << 52);
+  return __longlong_as_double(bits | (neg ? (1ll << 63) : 0ll));
+}
+
+// Fast path for r ≤ 12 (M < 2^112) in 32- and 64-bit words.  With
+// S = Σ_k c_k W_k (≡ X mod M) and W_k/M = y_k/m_k:
+//  * Y = Σ c_k F_k mod 2^64, read as a signed word, is 2^64·X/M up to
+//    Σ|c_k|/2 units, as long as X/M is not within that of ±1/2;
+//  * q = (S - X)/M is the integer nearest to Σ c_k g_k/2^31 - Y/2^64
+//    (evaluated in units of 2^-11);
+//  * L = X mod 2^64 = Σ c_k (W_k mod 2^64) - q·(M mod 2^64), exactly;
+//  * H = ⌊X/2^64⌋ is the integer nearest to Y·round(M/2^51)/2^77 - L/2^64,
+//    from three 32×32 products (the dropped low product is below 1 unit).
+// For |c_k| < m_k the error of the estimate of X/2^64 is below 2^-3.4, so H
+// is exact.  When |Y| is within about 2^52 of 2^63 (X within M/2^12 of
+// ±M/2, which products bounded by Eq. M-bound never reach) the function
+// returns false and the caller takes Garner's algorithm.
 template <int R>
-__global__ void __launch_bounds__(kCrtThreads) crt_kernel(int64_t m, int64_t n, const __grid_constant__ Oz2Moduli mods,
-                                                          const int16_t* __restrict__ res, int64_t ldr,
-                                                          const int* __restrict__ d, const int* __restrict__ e,
-                                                          double* __restrict__ C, int64_t ldc, int vec_in) {
-  __shared__ double tile[kCrtRows][kCrtCols + 1];
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const uint32_t tiles_m = static_cast<uint32_t>((m + kCrtRows - 1) / kCrtRows);
-  const uint32_t ntiles = tiles_m * static_cast<uint32_t>((n + kCrtCols - 1) / kCrtCols);
-  const size_t mstride = static_cast<size_t>(m) * ldr;
-  for (uint32_t t = blockIdx.x; t < ntiles; t += gridDim.x) {
-    const int64_t r0 = static_cast<int64_t>(t % tiles_m) * kCrtRows, c0 = static_cast<int64_t>(t / tiles_m) * kCrtCols;
-    const int64_t cb = c0 + 4 * lane;
-    int ecol[4];
+__device__ __forceinline__ bool crt_value_w64(const int (&c)[R], int E, const Oz2Moduli& mods, double& out) {
+  long long y0 = 0, l0 = 0, g0 = 0;
+  uint32_t y1 = 0, l1 = 0;
 #pragma unroll
-    for (int u = 0; u < 4; ++u) ecol[u] = cb + u < n ? e[cb + u] : 0;
-    for (int s = 0; s < kCrtRows / 8; ++s) {
-      const int lr = warp + 8 * s;
-      const int64_t row = r0 + lr;
-      if (row >= m) continue;
-      const int dr = d[row];
-      const int16_t* p = res + row * ldr + cb;
-      uint32_t lo[R], hi[R];  // residues of columns (cb, cb+1) and (cb+2, cb+3), packed int16 pairs
-      if (vec_in && cb + 3 < n) {
+  for (int k = 0; k < R; ++k) {
+    mad_word(c[k], mods.crt_fl[k], mods.crt_fh[k], y0, y1);
+    mad_word(c[k], mods.crt_wl[k], mods.crt_wh[k], l0, l1);
+    g0 += static_cast<long long>(c[k]) * mods.crt_g[k];
+  }
+  const uint32_t yl = static_cast<uint32_t>(y0);
+  const int yh = static_cast<int>(static_cast<uint32_t>(static_cast<u64>(y0) >> 32) + y1);
+  if ((yh ^ (yh >> 31)) >= 0x7FF00000) return false;
+  const int q = (static_cast<int>(g0 >> 20) - (yh >> 21) + 1024) >> 11;
+  l0 -= static_cast<long long>(q) * mods.crt_ml;
+  l1 -= static_cast<uint32_t>(q) * static_cast<uint32_t>(mods.crt_mlh);
+  const u64 L = static_cast<u64>(l0) + (static_cast<u64>(l1) << 32);
+  const long long mid = static_cast<long long>(yh) * mods.crt_m51l +
+                        static_cast<long long>(static_cast<u64>(yl) * static_cast<uint32_t>(mods.crt_m51h));
+  const long long zh = static_cast<long long>(yh) * mods.crt_m51h + (mid >> 32);  // ≈ X/2^51
+  const long long H = (zh - static_cast<long long>(static_cast<uint32_t>(L >> 51)) + 4096) >> 13;
+  out = finish_words(H, L, E);
+  return true;
+}
+
+constexpr int kCrtThreads = 256;
+constexpr long long kCrtSentinel = 0x7FF4DEAD0BADF00Dll;  // a NaN the reconstruction never produces
+
+template <int R>
+__device__ __forceinline__ bool crt_fast(const int (&c)[R], int E, const Oz2Moduli& mods, double& out) {
+  if constexpr (R <= 12)
+    return crt_value_w64<R>(c, E, mods, out);
+  else
+    return crt_value_fast<R>(c, E, mods, out);
+}
+
+// Resident blocks per SM the register budget is sized for: the two-word
+// path fits 64 registers up to r = 10; larger r gets more registers.
+template <int R>
+constexpr int crt_min_blocks() {
+  return R <= 10 ? 4 : (R <= 12 ? 3 : 2);
+}
+
+template <int R>
+__global__ void __launch_bounds__(kCrtThreads, crt_min_blocks<R>())
+    crt_kernel(int64_t m, int64_t n, const __grid_constant__ Oz2Moduli mods, const int16_t* __restrict__ res,
+               int64_t ldr, const int* __restrict__ d, const int* __restrict__ e, double* __restrict__ C,
+               int64_t ldc, int vec_in, int vec_out) {
+  const int64_t row = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) * 2;
+  if (row >= m) return;
+  const bool pair = row + 1 < m;
+  const size_t mstride = static_cast<size_t>(n) * ldr;
+  const int d0 = d[row], d1 = pair ? d[row + 1] : 0;
+  const int16_t* pbase = res + row;
+  double* cbase = C + row;
+  const int64_t step = gridDim.y;
+  // Two rows' residues of one column, packed (row in the low half).
+  auto load_words = [&](int64_t col, uint32_t (&w)[R]) {
+    const int16_t* p = pbase + col * ldr;
+    if (vec_in && pair) {
 #pragma unroll
-        for (int k = 0; k < R; ++k) {
-          const uint2 q = __ldg(reinterpret_cast<const uint2*>(p + k * mstride));
-          lo[k] = q.x;
-          hi[k] = q.y;
-        }
-      } else {
+      for (int k = 0; k < R; ++k) w[k] = __ldg(reinterpret_cast<const uint32_t*>(p + k * mstride));
+    } else {
 #pragma unroll
-        for (int k = 0; k < R; ++k) {
-          uint32_t w4[4];
-#pragma unroll
-          for (int u = 0; u < 4; ++u) w4[u] = cb + u < n ? static_cast<uint16_t>(p[k * mstride + u]) : 0u;
-          lo[k] = w4[0] | (w4[1] << 16);
-          hi[k] = w4[2] | (w4[3] << 16);
-        }
-      }
-#pragma unroll 1
-      for (int u = 0; u < 4; ++u) {
-        int c[R];
-#pragma unroll
-        for (int k = 0; k < R; ++k) {
-          const uint32_t w = u < 2 ? lo[k] : hi[k];
-          c[k] = static_cast<int>(static_cast<int16_t>((u & 1) ? (w >> 16) : (w & 0xFFFFu)));
-        }
-        const int eu = u == 0 ? ecol[0] : u == 1 ? ecol[1] : u == 2 ? ecol[2] : ecol[3];
-        double val;
-        if (!crt_value_fast<R>(c, -(dr + eu), mods, val)) val = crt_value<R>(c, -(dr + eu), mods);
-        tile[lr][4 * lane + u] = val;
-      }
+      for (int k = 0; k < R; ++k)
+        w[k] = static_cast<uint16_t>(p[k * mstride]) | (pair ? static_cast<uint32_t>(p[k * mstride + 1]) << 16 : 0u);
     }
-    __syncthreads();
-    // Column segments of 32 rows (256 bytes) per warp.
-    const int64_t row = r0 + lane;
-    for (int cc = warp; cc < kCrtCols; cc += kCrtThreads / 32) {
-      const int64_t col = c0 + cc;
-      if (col < n && row < m) C[row + col * ldc] = tile[lane][cc];
+  };
+  uint32_t nw[R];
+  int nec = 0;
+  if (static_cast<int64_t>(blockIdx.y) < n) {
+    load_words(blockIdx.y, nw);
+    nec = __ldg(e + blockIdx.y);
+  }
+  int pending = 0;
+  for (int64_t col = blockIdx.y; col < n; col += step) {
+    uint32_t w[R];
+#pragma unroll
+    for (int k = 0; k < R; ++k) w[k] = nw[k];
+    const int ec = nec;
+    if (col + step < n) {
+      load_words(col + step, nw);
+      nec = __ldg(e + col + step);
     }
-    __syncthreads();
+    double v[2];
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+      int c[R];
+#pragma unroll
+      for (int k = 0; k < R; ++k)
+        c[k] = u ? (static_cast<int>(w[k]) >> 16) : static_cast<int>(static_cast<int16_t>(w[k] & 0xFFFFu));
+      double val;
+      if (!crt_fast<R>(c, -((u ? d1 : d0) + ec), mods, val)) {
+        val = __longlong_as_double(kCrtSentinel);
+        ++pending;
+      }
+      v[u] = val;
+    }
+    double* out = cbase + col * ldc;
+    if (vec_out && pair) {
+      *reinterpret_cast<double2*>(out) = make_double2(v[0], v[1]);
+    } else {
+      out[0] = v[0];
+      if (pair) out[1] = v[1];
+    }
+  }
+  if (pending == 0) return;
+  // Outputs the fast path left to Garner's algorithm (this thread's own).
+  for (int64_t col = blockIdx.y; col < n; col += step) {
+    for (int u = 0; u < (pair ? 2 : 1); ++u) {
+      double* q = cbase + col * ldc + u;
+      if (__double_as_longlong(*q) != kCrtSentinel) continue;
+      const int16_t* p = pbase + col * ldr + u;
+      int c[R];
+#pragma unroll
+      for (int k = 0; k < R; ++k) c[k] = p[k * mstride];
+      *q = crt_value<R>(c, -((u ? d1 : d0) + __ldg(e + col)), mods);
+    }
   }
 }
 
 template <int R>
-static void launch_crt_r(int grid, cudaStream_t st, int64_t m, int64_t n, const Oz2Moduli& mods, const int16_t* res,
-                         int64_t ldr, const int32_t* d, const int32_t* e, double* C, int64_t ldc, int vi) {
-  crt_kernel<R><<<grid, kCrtThreads, 0, st>>>(m, n, mods, res, ldr, d, e, C, ldc, vi);
+static void launch_crt_r(dim3 grid, cudaStream_t st, int64_t m, int64_t n, const Oz2Moduli& mods, const int16_t* res,
+                         int64_t ldr, const int32_t* d, const int32_t* e, double* C, int64_t ldc, int vi, int vo) {
+  crt_kernel<R><<<grid, kCrtThreads, 0, st>>>(m, n, mods, res, ldr, d, e, C, ldc, vi, vo);
 }
 
 cudaError_t launch_reconstruct(int64_t m, int64_t n, const Oz2Moduli& mods, const int16_t* residues,
                                int64_t ldr, const int32_t* d, const int32_t* e, double* C, int64_t ldc,
                                cudaStream_t st) {
   if (m == 0 || n == 0) return cudaSuccess;
-  const int64_t tiles = ((m + kCrtRows - 1) / kCrtRows) * ((n + kCrtCols - 1) / kCrtCols);
   int dev = 0, sms = 148;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  const int grid = static_cast<int>(tiles < 16LL * sms ? tiles : 16LL * sms);
-  const int vi = (ldr % 4 == 0) && (reinterpret_cast<uintptr_t>(residues) % 8 == 0);
+  // x: row pairs; y: columns strided over gridDim.y, about two waves of
+  // 4 resident blocks per SM in total.
+  const int64_t gx = ((m + 1) / 2 + kCrtThreads - 1) / kCrtThreads;
+  if (gx > 0x7FFFFFFF) return cudaErrorInvalidValue;
+  int64_t gy = (8LL * sms + gx - 1) / gx;
+  gy = gy < 1 ? 1 : gy;
+  gy = gy > n ? n : gy;
+  gy = gy > 65535 ? 65535 : gy;
+  const dim3 grid(static_cast<unsigned>(gx), static_cast<unsigned>(gy));
+  const int vi = (ldr % 2 == 0) && (reinterpret_cast<uintptr_t>(residues) % 4 == 0);
+  const int vo = (ldc % 2 == 0) && (reinterpret_cast<uintptr_t>(C) % 16 == 0);
   count_launch();
   switch (mods.r) {
 #define OZ2_CRT_CASE(R) \
   case R:               \
-    launch_crt_r<R>(grid, st, m, n, mods, residues, ldr, d, e, C, ldc, vi); \
+    launch_crt_r<R>(grid, st, m, n, mods, residues, ldr, d, e, C, ldc, vi, vo); \
     break;
     OZ2_CRT_CASE(1) OZ2_CRT_CASE(2) OZ2_CRT_CASE(3) OZ2_CRT_CASE(4) OZ2_CRT_CASE(5) OZ2_CRT_CASE(6)
     OZ2_CRT_CASE(7) OZ2_CRT_CASE(8) OZ2_CRT_CASE(9) OZ2_CRT_CASE(10) OZ2_CRT_CASE(11) OZ2_CRT_CASE(12)

@@ -86,10 +86,10 @@ __device__ __forceinline__ float i16_to_float(uint32_t bits16) {
 }
 
 struct EpiCtx {
-  int16_t* res;   // r × (m×n row-major, ld = n)
+  int16_t* res;   // r × (m×n column-major, ld = ldr ≥ m; matrix i at i·n·ldr)
   float* urow;
   Oz2Device* dev;
-  int64_t m, n;
+  int64_t m, n, ldr;
 };
 
 struct UnitMap {
@@ -277,7 +277,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     const int h = (warp - 2) >> 2;             // 64-column quarter of the tile
     const uint32_t lane_addr = tmem + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(64 * h);
     const uint32_t acc_empty_leader = mapa_shared(acc_empty, 0);
-    const bool vec_ok = (ctx.n % 8) == 0;
     uint32_t accph = 0;
     for (int64_t u = pair; u < um.nunits && ok; u += npairs) {
       int i;
@@ -290,7 +289,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       const float inv = 1.f / mf;
       const float sb = MODE == 0 ? static_cast<float>(mods.sq_base[i]) : 0.f;
       const float hi = MODE == 0 ? static_cast<float>(mods.m[i] - 1 - mods.m[i] / 2) : 0.f;
-      int16_t* rrow = MODE == 0 ? ctx.res + static_cast<size_t>(i) * ctx.m * ctx.n + row * ctx.n : nullptr;
+      // This thread's row of C^(i); column j at rrow[j·ldr] (a warp stores 32
+      // consecutive rows of one column, 64 contiguous bytes, per instruction).
+      int16_t* rrow = MODE == 0 ? ctx.res + static_cast<size_t>(i) * ctx.n * ctx.ldr + row : nullptr;
       const int64_t slab = slab_steps_of<MODE>(mods, i, ksteps);
       float rowmax = 0.f;
       for (int64_t kb0 = 0; kb0 < ksteps; kb0 += slab) {
@@ -309,48 +310,26 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
             for (int j = 0; j < 16; ++j) rowmax = fmaxf(rowmax, __uint_as_float(v0[j]));
           } else if (row < ctx.m) {
             const int64_t cc = col0 + c;
-            int16_t* dst = rrow + cc;
-            const bool full = vec_ok && cc + 16 <= ctx.n;
-            uint32_t prevw[8];
-            if (kb0 && full) {
+            int16_t* dst = rrow + cc * ctx.ldr;
+            const int ncol = ctx.n - cc < 16 ? static_cast<int>(ctx.n - cc) : 16;
+            if (ncol == 16 && !kb0) {  // the common case: a full chunk, first slab
 #pragma unroll
-              for (int t = 0; t < 2; ++t) {
-                const uint4 pv = reinterpret_cast<const uint4*>(dst)[t];
-                prevw[4 * t] = pv.x;
-                prevw[4 * t + 1] = pv.y;
-                prevw[4 * t + 2] = pv.z;
-                prevw[4 * t + 3] = pv.w;
+              for (int j = 0; j < 16; ++j) {
+                const float rj =
+                    combine_residue(__uint_as_float(v0[j]), __uint_as_float(v1[j]), square, sb, mf, inv, hi, 0.f);
+                *dst = static_cast<int16_t>(as_i16_bits(rj));
+                dst += ctx.ldr;
               }
             } else {
+              float prev[16];
 #pragma unroll
-              for (int t = 0; t < 8; ++t) {
-                uint32_t a = 0, b = 0;
-                if (kb0 && cc + 2 * t < ctx.n) a = static_cast<uint16_t>(dst[2 * t]);
-                if (kb0 && cc + 2 * t + 1 < ctx.n) b = static_cast<uint16_t>(dst[2 * t + 1]);
-                prevw[t] = a | (b << 16);
-              }
-            }
-            uint32_t outw[8];
+              for (int j = 0; j < 16; ++j)
+                prev[j] = (kb0 && j < ncol) ? i16_to_float(static_cast<uint16_t>(dst[j * ctx.ldr])) : 0.f;
 #pragma unroll
-            for (int t = 0; t < 8; ++t) {
-              const float p0 = kb0 ? i16_to_float(prevw[t] & 0xFFFFu) : 0.f;
-              const float p1 = kb0 ? i16_to_float(prevw[t] >> 16) : 0.f;
-              const float r0 = combine_residue(__uint_as_float(v0[2 * t]), __uint_as_float(v1[2 * t]), square, sb, mf,
-                                               inv, hi, p0);
-              const float r1 = combine_residue(__uint_as_float(v0[2 * t + 1]), __uint_as_float(v1[2 * t + 1]), square,
-                                               sb, mf, inv, hi, p1);
-              outw[t] = as_i16_bits(r0) | (as_i16_bits(r1) << 16);
-            }
-            if (full) {
-#pragma unroll
-              for (int t = 0; t < 2; ++t)
-                reinterpret_cast<uint4*>(dst)[t] =
-                    make_uint4(outw[4 * t], outw[4 * t + 1], outw[4 * t + 2], outw[4 * t + 3]);
-            } else {
-#pragma unroll
-              for (int t = 0; t < 8; ++t) {
-                if (cc + 2 * t < ctx.n) dst[2 * t] = static_cast<int16_t>(outw[t] & 0xFFFFu);
-                if (cc + 2 * t + 1 < ctx.n) dst[2 * t + 1] = static_cast<int16_t>(outw[t] >> 16);
+              for (int j = 0; j < 16; ++j) {
+                const float rj = combine_residue(__uint_as_float(v0[j]), __uint_as_float(v1[j]), square, sb, mf, inv,
+                                                 hi, prev[j]);
+                if (j < ncol) dst[j * ctx.ldr] = static_cast<int16_t>(as_i16_bits(rj));
               }
             }
           }
@@ -430,7 +409,7 @@ __global__ void plane_gemm_simt_kernel(const uint8_t* __restrict__ pa, const uin
       }
       res = combine_residue(a0, a1, square, static_cast<float>(mods.sq_base[i]), mf, inv, hi, res);
     }
-    ctx.res[static_cast<size_t>(i) * ctx.m * ctx.n + row * ctx.n + col] = static_cast<int16_t>(res);
+    ctx.res[static_cast<size_t>(i) * ctx.n * ctx.ldr + col * ctx.ldr + row] = static_cast<int16_t>(res);
   }
 }
 
@@ -483,9 +462,9 @@ static int num_sms() {
 //       2 residues (SIMT reference), 3 magnitude (SIMT reference).
 cudaError_t launch_plane_gemm(int64_t m, int64_t n, int64_t k_pad, const Oz2Moduli& mods,
                               const uint8_t* planes_a, const uint8_t* planes_b, int mode,
-                              int16_t* residues, float* urow, Oz2Device* dev, cudaStream_t st) {
+                              int16_t* residues, int64_t ldr, float* urow, Oz2Device* dev, cudaStream_t st) {
   if (m == 0 || n == 0) return cudaSuccess;
-  EpiCtx ctx{residues, urow, dev, m, n};
+  EpiCtx ctx{residues, urow, dev, m, n, ldr};
   if (mode >= 2) {
     dim3 g(static_cast<unsigned>((m + 127) / 128), static_cast<unsigned>(n));
     count_launch();

@@ -119,6 +119,13 @@ static int bitlen3(const u64 (&x)[3]) {
   return 0;
 }
 
+// v = hi·2^32 + lo (mod 2^64) with lo the low word read as a signed integer.
+static void split_signed_low(u64 v, int* lo, int* hi) {
+  const int l = static_cast<int>(static_cast<uint32_t>(v));
+  *lo = l;
+  *hi = static_cast<int>(static_cast<uint32_t>((v - static_cast<u64>(static_cast<long long>(l))) >> 32));
+}
+
 static Oz2Moduli build_moduli(int r, int quant) {
   Oz2Moduli c;
   std::memset(&c, 0, sizeof(c));
@@ -178,10 +185,18 @@ static Oz2Moduli build_moduli(int r, int quant) {
     for (int t = 0; t < 5; ++t) c.crtw[k][t] = W[t];
     c.crtf[k] = static_cast<uint32_t>(((static_cast<u64>(y) << 32) + static_cast<u64>(mk / 2)) / static_cast<u64>(mk));
     c.coff[k] = mk * ((32768 + mk - 1) / mk);
+    // Two-word constants: y/m < 1 - 1/m, so both roundings stay below 2^64 and 2^31.
+    const unsigned __int128 fy = ((static_cast<unsigned __int128>(y) << 64) + static_cast<unsigned>(mk / 2)) / mk;
+    split_signed_low(static_cast<u64>(fy), &c.crt_fl[k], &c.crt_fh[k]);
+    split_signed_low(static_cast<u64>(W[0]) | (static_cast<u64>(W[1]) << 32), &c.crt_wl[k], &c.crt_wh[k]);
+    c.crt_g[k] = static_cast<int>(((static_cast<u64>(y) << 31) + static_cast<u64>(mk / 2)) / static_cast<u64>(mk));
   }
   u64 M[3] = {1, 0, 0};
   for (int i = 0; i < r; ++i) mul3(M, static_cast<u64>(kModuliAll[i]));
   for (int i = 0; i < 3; ++i) c.M[i] = M[i];
+  split_signed_low(M[0], &c.crt_ml, &c.crt_mlh);
+  // round(M/2^51), below 2^61 while M < 2^112 (r ≤ 12, the only use).
+  split_signed_low(((M[0] >> 51) | (M[1] << 13)) + ((M[0] >> 50) & 1), &c.crt_m51l, &c.crt_m51h);
   // ⌈M/2⌉ = (M + 1) >> 1
   u64 Mp[3] = {M[0] + 1, M[1] + (M[0] + 1 == 0), M[2]};
   c.Mhalf[0] = (Mp[0] >> 1) | (Mp[1] << 63);
@@ -307,10 +322,12 @@ static void compute_layout(int64_t m, int64_t n, int64_t k, int r, oz2_ws_layout
   L->mag_b = take(static_cast<size_t>(n) * k_pad);
   L->planes_a = take(static_cast<size_t>(planes) * m * k_pad);
   L->planes_b = take(static_cast<size_t>(planes) * n * k_pad);
-  L->residues = take(2 * static_cast<size_t>(r) * m * n);
+  const int64_t res_ld = (m + 7) / 8 * 8;  // 16-byte columns
+  L->residues = take(2 * static_cast<size_t>(r) * n * res_ld);
   L->total = off;
   L->k_pad = k_pad;
   L->num_planes = planes;
+  L->res_ld = res_ld;
 }
 
 static int check_sizes(int64_t m, int64_t n, int64_t k, int64_t lda, int64_t ldb, int64_t ldc) {
@@ -435,7 +452,7 @@ int oz2_dgemm_ex(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, 
       err = launch_magnitude_planes(m, n, k, A, lda, B, ldb, ra, cb, rf, cf, mag_a, mag_b, s);
     mark(2);
     if (err == cudaSuccess)
-      err = launch_plane_gemm(m, n, L.k_pad, mods, mag_a, mag_b, simt ? 3 : 1, nullptr, urow, ds->status, s);
+      err = launch_plane_gemm(m, n, L.k_pad, mods, mag_a, mag_b, simt ? 3 : 1, nullptr, 0, urow, ds->status, s);
     mark(3);
   } else {
     mark(2);
@@ -447,9 +464,9 @@ int oz2_dgemm_ex(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, 
     err = launch_deconstruct(m, n, k, mods, ds->table_a, ds->table_b, A, lda, B, ldb, d, e, rf, cf, quant, pa, pb, s);
   mark(5);
   if (err == cudaSuccess)
-    err = launch_plane_gemm(m, n, L.k_pad, mods, pa, pb, simt ? 2 : 0, res, nullptr, ds->status, s);
+    err = launch_plane_gemm(m, n, L.k_pad, mods, pa, pb, simt ? 2 : 0, res, L.res_ld, nullptr, ds->status, s);
   mark(6);
-  if (err == cudaSuccess) err = launch_reconstruct(m, n, mods, res, n, d, e, C, ldc, s);
+  if (err == cudaSuccess) err = launch_reconstruct(m, n, mods, res, L.res_ld, d, e, C, ldc, s);
   mark(7);
   if (err == cudaSuccess) err = launch_fallback_lists(m, n, k, A, lda, B, ldb, rf, cf, misc, C, ldc, s);
   mark(8);
@@ -608,7 +625,8 @@ int oz2_scale(int64_t m, int64_t n, int64_t k, int num_moduli, const double* A, 
   if (scale == OZ2_SCALE_R2) {
     if (err == cudaSuccess)
       err = launch_magnitude_planes(m, n, k, A, lda, B, ldb, ra, cb, row_flag, col_flag, mag_a, mag_b, s);
-    if (err == cudaSuccess) err = launch_plane_gemm(m, n, k_pad, mods, mag_a, mag_b, 1, nullptr, urow, ds->status, s);
+    if (err == cudaSuccess)
+      err = launch_plane_gemm(m, n, k_pad, mods, mag_a, mag_b, 1, nullptr, 0, urow, ds->status, s);
   }
   if (err == cudaSuccess)
     err = launch_choose_scales(m, n, k, mods, scale, urow, ra, cb, row_flag, col_flag, d, e, ds->status, s);
@@ -630,8 +648,8 @@ int oz2_deconstruct(int64_t m, int64_t n, int64_t k, int num_moduli, const doubl
 }
 
 int oz2_residue_gemm(int64_t m, int64_t n, int64_t k, int num_moduli, const uint8_t* planes_a,
-                     const uint8_t* planes_b, int16_t* residues, void* stream) {
-  if (m <= 0 || n <= 0 || k <= 0 || !planes_a || !planes_b || !residues) return OZ2_ERR_INVALID_ARG;
+                     const uint8_t* planes_b, int16_t* residues, int64_t ldr, void* stream) {
+  if (m <= 0 || n <= 0 || k <= 0 || !planes_a || !planes_b || !residues || ldr < m) return OZ2_ERR_INVALID_ARG;
   if (num_moduli < 1 || num_moduli > kMaxModuli) return OZ2_ERR_UNSUPPORTED_R;
   if (m >= (1LL << 31) || n >= (1LL << 31) || k > (1LL << 24)) return OZ2_ERR_UNSUPPORTED;
   DeviceState* ds = nullptr;
@@ -639,26 +657,26 @@ int oz2_residue_gemm(int64_t m, int64_t n, int64_t k, int num_moduli, const uint
   if (st) return st;
   const Oz2Moduli mods = build_moduli(num_moduli, OZ2_QUANT_TZ);
   const int64_t k_pad = (k + kKPad - 1) / kKPad * kKPad;
-  return to_status(launch_plane_gemm(m, n, k_pad, mods, planes_a, planes_b, 0, residues, nullptr, ds->status,
+  return to_status(launch_plane_gemm(m, n, k_pad, mods, planes_a, planes_b, 0, residues, ldr, nullptr, ds->status,
                                      static_cast<cudaStream_t>(stream)));
 }
 
 int oz2_residue_gemm_simt(int64_t m, int64_t n, int64_t k, int num_moduli, const uint8_t* planes_a,
-                          const uint8_t* planes_b, int16_t* residues, void* stream) {
-  if (m <= 0 || n <= 0 || k <= 0 || !planes_a || !planes_b || !residues) return OZ2_ERR_INVALID_ARG;
+                          const uint8_t* planes_b, int16_t* residues, int64_t ldr, void* stream) {
+  if (m <= 0 || n <= 0 || k <= 0 || !planes_a || !planes_b || !residues || ldr < m) return OZ2_ERR_INVALID_ARG;
   if (num_moduli < 1 || num_moduli > kMaxModuli) return OZ2_ERR_UNSUPPORTED_R;
   DeviceState* ds = nullptr;
   int st = device_state(&ds);
   if (st) return st;
   const Oz2Moduli mods = build_moduli(num_moduli, OZ2_QUANT_TZ);
   const int64_t k_pad = (k + kKPad - 1) / kKPad * kKPad;
-  return to_status(launch_plane_gemm(m, n, k_pad, mods, planes_a, planes_b, 2, residues, nullptr, ds->status,
+  return to_status(launch_plane_gemm(m, n, k_pad, mods, planes_a, planes_b, 2, residues, ldr, nullptr, ds->status,
                                      static_cast<cudaStream_t>(stream)));
 }
 
 int oz2_reconstruct(int64_t m, int64_t n, int num_moduli, const int16_t* residues, int64_t ldr, const int32_t* d,
                     const int32_t* e, double* C, int64_t ldc, void* stream) {
-  if (m < 0 || n < 0 || ldr < std::max<int64_t>(1, n) || ldc < std::max<int64_t>(1, m)) return OZ2_ERR_INVALID_ARG;
+  if (m < 0 || n < 0 || ldr < std::max<int64_t>(1, m) || ldc < std::max<int64_t>(1, m)) return OZ2_ERR_INVALID_ARG;
   if (num_moduli < 1 || num_moduli > kMaxModuli) return OZ2_ERR_UNSUPPORTED_R;
   if (m && n && (!residues || !d || !e || !C)) return OZ2_ERR_INVALID_ARG;
   const Oz2Moduli mods = build_moduli(num_moduli, OZ2_QUANT_TZ);

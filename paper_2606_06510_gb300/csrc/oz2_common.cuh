@@ -108,6 +108,16 @@ struct Oz2Moduli {
   uint32_t crtw[kMaxModuli][5];
   uint32_t crtf[kMaxModuli];
   int coff[kMaxModuli];
+  // Two-word direct CRT (r ≤ 12, M < 2^112), for signed 32×32→64-bit
+  // multiply-adds: F_k = round(2^64·y_k/m_k) mod 2^64 = fh·2^32 + fl and
+  // W_k mod 2^64 = wh·2^32 + wl, each with a signed low word;
+  // g_k = round(2^31·y_k/m_k); M mod 2^64 = mlh·2^32 + ml and
+  // round(M/2^51) = m51h·2^32 + m51l (ml, m51l signed).
+  int crt_fl[kMaxModuli], crt_fh[kMaxModuli];
+  int crt_wl[kMaxModuli], crt_wh[kMaxModuli];
+  int crt_g[kMaxModuli];
+  int crt_ml, crt_mlh;
+  int crt_m51l, crt_m51h;
   int table_entries;            // Σ m_i
 };
 
@@ -379,7 +389,7 @@ cudaError_t launch_deconstruct(int64_t m, int64_t n, int64_t k, const Oz2Moduli&
                                uint8_t* planes_a, uint8_t* planes_b, cudaStream_t st);
 cudaError_t launch_plane_gemm(int64_t m, int64_t n, int64_t k_pad, const Oz2Moduli& mods,
                               const uint8_t* planes_a, const uint8_t* planes_b, int mode,
-                              int16_t* residues, float* urow, Oz2Device* dev, cudaStream_t st);
+                              int16_t* residues, int64_t ldr, float* urow, Oz2Device* dev, cudaStream_t st);
 cudaError_t launch_reconstruct(int64_t m, int64_t n, const Oz2Moduli& mods,
                                const int16_t* residues, int64_t ldr, const int32_t* d,
                                const int32_t* e, double* C, int64_t ldc, cudaStream_t st);

@@ -50,6 +50,9 @@ def test_host_argument_errors(oz):
     assert L.oz2_dgemm_ex(8, 8, 8, 1, 8, 1, 8, 1, 8, 12, 5, 0, 0, null, 0, null) == -1
     assert L.oz2_dgemm_ex(8, 8, 8, 1, 8, 1, 8, 1, 8, 12, 0, 0, 0, null, 0, null) == -3
     assert L.oz2_dgemm_ex(8, 8, 8, 1, 8, 1, 8, 1, 8, 12, 0, 0, 0, 3, 1 << 30, null) == -3
+    # stage entries: residue leading dimension below m
+    assert L.oz2_residue_gemm(8, 8, 8, 12, 1, 1, 1, 7, null) == -1
+    assert L.oz2_reconstruct(8, 8, 12, 1, 7, 1, 1, 1, 8, null) == -1
 
 
 def test_layout_queries(oz):
@@ -63,5 +66,6 @@ def test_layout_queries(oz):
     offs = [L[k] for k in keys]
     assert offs == sorted(offs) and all(o % 256 == 0 for o in offs)
     assert L["planes_b"] - L["planes_a"] >= 30 * 300 * 256
-    assert L["total"] - L["residues"] >= 2 * 12 * 300 * 200
+    assert L["res_ld"] == 304 and L["total"] - L["residues"] >= 2 * 12 * 304 * 200
+    assert oz.oz2_workspace_layout(301, 5, 1, 3)["res_ld"] == 304
     assert oz.oz2_workspace_size(300, 200, 129, 12) == L["total"]

@@ -1,0 +1,95 @@
+"""Error budget of the reconstruction's two-word fast path (r ≤ 12).
+
+The CUDA reconstruction finds X from 64-bit fixed-point sums: Y = Σ c_k F_k
+mod 2^64 with F_k = round(2^64·y_k/m_k) approximates 2^64·X/M, and
+H = ⌊X/2^64⌋ is recovered from Y·round(M/2^49)/2^113.  These CPU tests check,
+with exact rational arithmetic on constants built here from their
+definitions, that the worst case over all residues with |c_k| < m_k keeps
+the error of that estimate well below the 1/2 that rounding H tolerates, and
+that the quotient estimate keeps its margin too.  They also run the
+word-level arithmetic on Python integers for random and extreme X.
+"""
+from fractions import Fraction
+import random
+
+import pytest
+
+from oracle import ozaki2 as orc
+
+
+def constants(r):
+    mods = orc.moduli(r)
+    M = 1
+    for m in mods:
+        M *= m
+    out = []
+    for m in mods:
+        Mk = M // m
+        y = pow(Mk % m, -1, m)
+        F = ((y << 64) + m // 2) // m
+        g = ((y << 31) + m // 2) // m
+        out.append((m, y, Mk * y, F, g))
+    return M, mods, out
+
+
+@pytest.mark.parametrize("r", range(1, 13))
+def test_fraction_error_budget(r):
+    M, mods, cs = constants(r)
+    assert M < 2 ** 112
+    mh = (M + (1 << 48)) >> 49
+    assert mh < 2 ** 63
+    # |Y - 2^64·X/M| ≤ Σ |c_k|·|F_k - 2^64 y_k/m_k| with |c_k| ≤ m_k - 1.
+    err_y = sum((m - 1) * abs(Fraction(F) - Fraction(y << 64, m)) for m, y, _, F, _ in cs)
+    assert err_y <= Fraction(1, 2) * sum(m - 1 for m in mods)
+    # H estimate in units of 2^64: Y error scaled by M/2^64, plus the rounding
+    # of M/2^49 (|Y| < 2^63), the floor of the high product and of L/2^49.
+    err_h = err_y * Fraction(M, 2 ** 64) / 2 ** 64 + Fraction(2 ** 63, 2 ** 64) * Fraction(1, 2) / 2 ** 15 \
+        + Fraction(2, 2 ** 15)
+    assert err_h < Fraction(1, 8), float(err_h)
+    # Quotient estimate Σ c_k g_k/2^31 - Y/2^64: error well below 1/2.
+    err_q = sum((m - 1) * abs(Fraction(g) - Fraction(y << 31, m)) for m, y, _, _, g in cs) / 2 ** 31 \
+        + (err_y + 1) / 2 ** 64 + Fraction(1, 2 ** 31)
+    assert err_q < Fraction(1, 2 ** 12), float(err_q)
+    # The margin in Y (2^52) is far above its error.
+    assert err_y < 2 ** 40
+
+
+def word_path(c, r):
+    """The fast path's word arithmetic on Python integers (two's complement
+    words emulated with masks); returns X, or None where it defers."""
+    M, mods, cs = constants(r)
+    mask = (1 << 64) - 1
+    Y = sum(ck * F for ck, (_, _, _, F, _) in zip(c, cs)) & mask
+    Ys = Y - (1 << 64) if Y >> 63 else Y
+    if abs(Ys if Ys >= 0 else ~Ys) >= (1 << 63) - (1 << 52):
+        return None
+    g0 = sum(ck * g for ck, (_, _, _, _, g) in zip(c, cs))
+    q = (g0 - (Ys >> 33) + (1 << 30)) >> 31
+    L = (sum(ck * W for ck, (_, _, W, _, _) in zip(c, cs)) - q * M) & mask
+    mh = (M + (1 << 48)) >> 49
+    zh = (Ys * mh) >> 64
+    H = (zh - (L >> 49) + (1 << 14)) >> 15
+    return H * 2 ** 64 + L
+
+
+@pytest.mark.parametrize("r", [1, 4, 8, 11, 12])
+def test_word_path_recovers_x(r):
+    M, mods, _ = constants(r)
+    rng = random.Random(r)
+    lo, hi = -(M // 2), M - M // 2 - 1
+    xs = [0, 1, -1, lo, hi, lo + (M >> 12) + 1, hi - (M >> 12) - 1]
+    xs += [rng.randrange(lo, hi + 1) for _ in range(300)]
+    xs += [rng.randrange(max(lo, -(1 << 64)), min(hi, 1 << 64) + 1) for _ in range(100)]
+    deferred = 0
+    for x in xs:
+        c = [int(orc.centred(x % m, m)) for m in mods]
+        # also a non-centred representative with |c| < m
+        c2 = [ck + m if ck < 0 else ck - m if ck > 0 else ck for ck, m in zip(c, mods)]
+        for cc in (c, c2):
+            got = word_path(cc, r)
+            if got is None:
+                deferred += 1
+                assert abs(x) > M // 2 - (M >> 11)
+            else:
+                assert got == x, (r, x)
+    assert deferred <= 8

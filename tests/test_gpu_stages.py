@@ -188,22 +188,30 @@ def test_residue_gemm_accumulator_extremes(oz):
 def test_reconstruct(oz):
     import torch
     rng = np.random.default_rng(41)
-    for r in (1, 2, 7, 12, 13, 16):
+    cases = [(r, 70, 33, None) for r in (1, 2, 7, 12, 13, 16)]
+    cases += [(12, 71, 5, 74), (12, 71, 6, 75), (13, 9, 7, 9), (5, 1, 3, 1)]  # odd rows, odd/even ld
+    for r, m, n, ldr in cases:
         mods = orc.moduli(r)
-        m, n = 70, 33
         R = np.stack([orc.centred(rng.integers(0, mi, size=(m, n)), mi) for mi in mods])
         R[:, 0, 0] = 0
         d = rng.integers(40, 80, size=m)
         e = rng.integers(40, 80, size=n)
-        d[1], d[2], d[3] = 1100, 1180, -1100            # subnormal, underflow, overflow rows
-        res = torch.from_numpy(np.ascontiguousarray(R).astype(np.int16)).cuda()
+        if m > 3:
+            d[1], d[2], d[3] = 1100, 1180, -1100            # subnormal, underflow, overflow rows
+        if ldr is None:
+            res = torch.from_numpy(np.ascontiguousarray(R).astype(np.int16)).cuda()
+        else:   # column-major storage with the given leading dimension
+            buf = torch.full((r, n, ldr), 777, dtype=torch.int16)
+            buf[:, :, :m] = torch.from_numpy(R.transpose(0, 2, 1).astype(np.int16))
+            res = buf.cuda()[:, :, :m].transpose(1, 2)
+            assert res.stride() == (n * ldr, 1, ldr)
         C = oz.oz2_reconstruct(res, torch.from_numpy(d.astype(np.int32)).cuda(),
                                torch.from_numpy(e.astype(np.int32)).cuda(), m, n, r).cpu().numpy()
         X = orc.garner_value(R, mods)
         for i in range(m):
             for j in range(n):
                 want = orc.unscale_one(int(X[i, j]), -int(d[i]) - int(e[j]))
-                assert C[i, j] == want and np.signbit(C[i, j]) == np.signbit(want), (r, i, j)
+                assert C[i, j] == want and np.signbit(C[i, j]) == np.signbit(want), (r, m, n, i, j)
 
 
 def test_reconstruct_near_the_range_boundary(oz):
@@ -219,6 +227,10 @@ def test_reconstruct_near_the_range_boundary(oz):
         xs = [lo, lo + 1, hi, hi - 1, 0, 1, -1]
         band = max(1, M >> 13)
         xs += [lo + rng.randrange(band) for _ in range(60)] + [hi - rng.randrange(band) for _ in range(60)]
+        # Either side of the fast path's margin (X within M/2^12 of ±M/2).
+        edge = M >> 12
+        xs += [lo + edge + rng.randrange(-band, band) for _ in range(40)]
+        xs += [hi - edge + rng.randrange(-band, band) for _ in range(40)]
         xs += [rng.randrange(lo, hi + 1) for _ in range(60)]
         m, n = len(xs), 3
         R = np.zeros((r, m, n), dtype=np.int64)
@@ -234,6 +246,34 @@ def test_reconstruct_near_the_range_boundary(oz):
             for j in range(n):
                 want = orc.unscale_one(x, -int(d[i]) - int(e[j]))
                 assert C[i, j] == want and np.signbit(C[i, j]) == np.signbit(want), (r, i, j)
+
+
+def test_reconstruct_other_representatives(oz):
+    """Residues in (-m_i, m_i) that are not the centred ones give the same
+    results as the centred ones (the reconstruction's input contract)."""
+    import torch
+    rng = np.random.default_rng(43)
+    for r in (5, 12, 13):
+        mods = orc.moduli(r)
+        m, n = 40, 36
+        R = np.stack([orc.centred(rng.integers(0, mi, size=(m, n)), mi) for mi in mods])
+        shift = rng.integers(0, 2, size=R.shape).astype(bool)
+        Ralt = R.copy()
+        for k, mk in enumerate(mods):
+            moved = np.where(R[k] < 0, R[k] + mk, np.where(R[k] > 0, R[k] - mk, 0))
+            Ralt[k] = np.where(shift[k], moved, R[k])
+            assert (np.abs(Ralt[k]) < mk).all()
+        d = rng.integers(40, 80, size=m)
+        e = rng.integers(40, 80, size=n)
+        dev_d = torch.from_numpy(d.astype(np.int32)).cuda()
+        dev_e = torch.from_numpy(e.astype(np.int32)).cuda()
+        C1 = oz.oz2_reconstruct(torch.from_numpy(R.astype(np.int16)).cuda(), dev_d, dev_e, m, n, r).cpu().numpy()
+        C2 = oz.oz2_reconstruct(torch.from_numpy(Ralt.astype(np.int16)).cuda(), dev_d, dev_e, m, n, r).cpu().numpy()
+        X = orc.garner_value(R, mods)
+        for i in range(m):
+            for j in range(n):
+                want = orc.unscale_one(int(X[i, j]), -int(d[i]) - int(e[j]))
+                assert C1[i, j] == want and C2[i, j] == want, (r, i, j)
 
 
 def test_fallback_rows_and_columns(oz):
