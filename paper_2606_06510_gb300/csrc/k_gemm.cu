@@ -17,8 +17,9 @@
 // accumulator merge of §2.5 "Accumulators").  Every K-slab (32768 squares,
 // 4096 nonsquare: Eq. accum-exact) the epilogue reads the accumulators and
 // forms  v = acc0 + s·acc1  or  v = 16·acc0 - 15·acc1  mod m, adds the
-// previous slab's residue and stores the centred residue as int16, row-major
-// (each thread owns one row and 16 consecutive columns: 16-byte stores).
+// previous slab's residue and stores the centred residue as int16,
+// column-major (each thread owns one row; a warp's store covers 32
+// consecutive rows of one column, 64 contiguous bytes).
 //
 // Pipeline: a stage is one (A plane, B plane) pair of 128-byte-deep tiles
 // (32 KiB per CTA), six stages.  Warp 0 of each CTA issues its CTA's TMA
@@ -202,12 +203,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     // ---------------- MMA issuer (leader CTA) ----------------
     if (leader && lane == 0) {
       constexpr uint32_t idesc = idesc_f8_f32(kTileM, kTileN);
-      uint32_t it = 0, accph = 0;
-      auto wait_full = [&](uint32_t j) {
-        return mbar_wait_bounded(full0 + 8 * (j % kStages), (j / kStages) & 1, kWaitLimit);
-      };
-      auto desc = [&](uint32_t j, int operand, int kk) {
-        return smem_desc_sw128(smem_u32(smem + (j % kStages) * kStageBytes + operand * kTileBytes) + kk * 32);
+      // Stage s, operand o, k-chunk kk: the descriptor of stage 0 plus the
+      // byte offset >> 4 (the start-address field has room: smem < 256 KiB).
+      const uint64_t desc0 = smem_desc_sw128(smem_u32(smem));
+      uint32_t st = 0, ph = 0, accph = 0;   // current stage and its full-barrier parity
+      auto next = [&](uint32_t& s_, uint32_t& p_) {
+        if (++s_ == kStages) {
+          s_ = 0;
+          p_ ^= 1;
+        }
       };
       for (int64_t u = pair; u < um.nunits && ok; u += npairs) {
         int i;
@@ -225,35 +229,43 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           for (int64_t kb = kb0; kb < kb1 && ok; ++kb) {
             const uint32_t first = kb == kb0 ? 0u : 1u;
             if (np == 2) {  // square: stages (d0,e0) and (d1,e1)
-              if (!wait_full(it) || !wait_full(it + 1)) {
+              uint32_t s1 = st, p1 = ph;
+              next(s1, p1);
+              if (!mbar_wait_bounded(full0 + 8 * st, ph, kWaitLimit) || !mbar_wait_bounded(full0 + 8 * s1, p1, kWaitLimit)) {
                 ok = false;
                 break;
               }
               tc_fence_after();
+              const uint64_t a0 = desc0 + st * (kStageBytes >> 4), b0 = a0 + (kTileBytes >> 4);
+              const uint64_t a1 = desc0 + s1 * (kStageBytes >> 4), b1 = a1 + (kTileBytes >> 4);
 #pragma unroll
               for (int kk = 0; kk < kBK / 32; ++kk) {
                 const uint32_t acc = kk ? 1u : first;
-                mma_f8_pair(tmem, desc(it, 0, kk), desc(it, 1, kk), idesc, acc);                   // d0·e0
-                mma_f8_pair(tmem + kAccCols, desc(it + 1, 0, kk), desc(it, 1, kk), idesc, acc);    // d1·e0
-                mma_f8_pair(tmem + kAccCols, desc(it, 0, kk), desc(it + 1, 1, kk), idesc, 1u);     // + d0·e1
+                mma_f8_pair(tmem, a0 + 2 * kk, b0 + 2 * kk, idesc, acc);                 // d0·e0
+                mma_f8_pair(tmem + kAccCols, a1 + 2 * kk, b0 + 2 * kk, idesc, acc);      // d1·e0
+                mma_f8_pair(tmem + kAccCols, a0 + 2 * kk, b1 + 2 * kk, idesc, 1u);       // + d0·e1
               }
-              mma_commit_pair_mc(empty0 + 8 * (it % kStages), 0x3);
-              mma_commit_pair_mc(empty0 + 8 * ((it + 1) % kStages), 0x3);
-              it += 2;
+              mma_commit_pair_mc(empty0 + 8 * st, 0x3);
+              mma_commit_pair_mc(empty0 + 8 * s1, 0x3);
+              st = s1;
+              ph = p1;
+              next(st, ph);
             } else {
-              for (int p = 0; p < np; ++p, ++it) {  // nonsquare: Σ·Σ → acc0; d0e0, -16 d1·e1 → acc1
-                if (!wait_full(it)) {
+              for (int p = 0; p < np; ++p) {  // nonsquare: Σ·Σ → acc0; d0e0, -16 d1·e1 → acc1
+                if (!mbar_wait_bounded(full0 + 8 * st, ph, kWaitLimit)) {
                   ok = false;
                   break;
                 }
                 tc_fence_after();
                 const uint32_t col = p == 0 ? 0u : kAccCols;
+                const uint64_t a = desc0 + st * (kStageBytes >> 4), b = a + (kTileBytes >> 4);
 #pragma unroll
                 for (int kk = 0; kk < kBK / 32; ++kk) {
                   const uint32_t acc = (kk || p == 2) ? 1u : first;
-                  mma_f8_pair(tmem + col, desc(it, 0, kk), desc(it, 1, kk), idesc, acc);
+                  mma_f8_pair(tmem + col, a + 2 * kk, b + 2 * kk, idesc, acc);
                 }
-                mma_commit_pair_mc(empty0 + 8 * (it % kStages), 0x3);
+                mma_commit_pair_mc(empty0 + 8 * st, 0x3);
+                next(st, ph);
               }
             }
           }
