@@ -62,7 +62,7 @@ def parse():
     p.add_argument("--steps", type=int, default=200)
     p.add_argument("--warmup", type=int, default=5)
     p.add_argument("--workload", default="dgemm_4096", choices=sorted(wl.WORKLOADS))
-    p.add_argument("--num-moduli", type=int, default=12)
+    p.add_argument("--num-moduli", type=int, default=None, help="default: the workload's FP64-grade r")
     p.add_argument("--impl", default="oz2", choices=["oz2", "reference"])
     p.add_argument("--no-sweep", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -180,7 +180,7 @@ def run_oz2(args):
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     w = wl.WORKLOADS[args.workload]
-    r = args.num_moduli
+    r = args.num_moduli or w.r
     A, B = wl.make_inputs(w)
     dA = oz.colmajor(torch.from_numpy(np.ascontiguousarray(A)).to(dev))
     dB = oz.colmajor(torch.from_numpy(np.ascontiguousarray(B)).to(dev))
@@ -345,7 +345,7 @@ def run_reference(args):
         return
     from oracle import ozaki2 as orc
     w = wl.WORKLOADS[args.workload]
-    r = args.num_moduli
+    r = args.num_moduli or w.r
     A, B = wl.make_inputs(w)
     t0 = time.perf_counter()
     prep = orc.prepare(A, B, r)
