@@ -79,6 +79,13 @@ __device__ __forceinline__ float combine_residue(float a0, float a1, bool square
   const float v = (square ? fmaf(s, r1, r0) : fmaf(16.f, r0, -15.f * r1)) + prev;
   return centred_small(v, m, inv_m, hi);
 }
+// The same for a short slab, where v itself is an integer below 2^24 and the
+// accumulators need no reduction before they are combined (see short_slab).
+__device__ __forceinline__ float combine_residue_short(float a0, float a1, bool square, float s, float m,
+                                                       float inv_m, float hi) {
+  const float v = square ? fmaf(s, a1, a0) : fmaf(16.f, a0, -15.f * a1);
+  return centred_small(loose_mod(v, m, inv_m), m, inv_m, hi);
+}
 // int16 encoding of an integer-valued float in [-2^15, 2^15).
 __device__ __forceinline__ uint32_t as_i16_bits(float r) { return __float_as_uint(r + kRoundMagic) & 0xFFFFu; }
 __device__ __forceinline__ float i16_to_float(uint32_t bits16) {
@@ -305,6 +312,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       // consecutive rows of one column, 64 contiguous bytes, per instruction).
       int16_t* rrow = MODE == 0 ? ctx.res + static_cast<size_t>(i) * ctx.n * ctx.ldr + row : nullptr;
       const int64_t slab = slab_steps_of<MODE>(mods, i, ksteps);
+      // Short slabs (K = 128·ksteps k-entries): v stays an integer below 2^24
+      // without reducing the accumulators first.  Square moduli (|d0e0| ≤ 256,
+      // |d1e0 + d0e1| ≤ 512, s ≤ 33): |v| ≤ K(256 + 33·512) < 2^24 for K ≤ 896.
+      // Nonsquare (|(d0+d1)(e0+e1)| ≤ 22², merged term ≤ 4095):
+      // |16·acc0 - 15·acc1| ≤ K(16·484 + 15·4095) < 2^24 for K ≤ 128.
+      const bool short_slab = MODE == 0 && ksteps <= (square ? 7 : 1);
       float rowmax = 0.f;
       for (int64_t kb0 = 0; kb0 < ksteps; kb0 += slab) {
         if (!mbar_wait_bounded(acc_full, accph, kWaitLimit)) {
@@ -324,7 +337,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
             const int64_t cc = col0 + c;
             int16_t* dst = rrow + cc * ctx.ldr;
             const int ncol = ctx.n - cc < 16 ? static_cast<int>(ctx.n - cc) : 16;
-            if (ncol == 16 && !kb0) {  // the common case: a full chunk, first slab
+            if (ncol == 16 && !kb0 && short_slab) {
+#pragma unroll
+              for (int j = 0; j < 16; ++j) {
+                const float rj =
+                    combine_residue_short(__uint_as_float(v0[j]), __uint_as_float(v1[j]), square, sb, mf, inv, hi);
+                *dst = static_cast<int16_t>(as_i16_bits(rj));
+                dst += ctx.ldr;
+              }
+            } else if (ncol == 16 && !kb0) {  // the common case: a full chunk, first slab
 #pragma unroll
               for (int j = 0; j < 16; ++j) {
                 const float rj =
