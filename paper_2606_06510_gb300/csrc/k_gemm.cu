@@ -16,10 +16,12 @@
 // (the A operand stores its last nonsquare plane pre-scaled by -2^b, the
 // accumulator merge of §2.5 "Accumulators").  Every K-slab (32768 squares,
 // 4096 nonsquare: Eq. accum-exact) the epilogue reads the accumulators and
-// forms  v = acc0 + s·acc1  or  v = 16·acc0 - 15·acc1  mod m, adds the
-// previous slab's residue and stores the centred residue as int16,
-// column-major (each thread owns one row; a warp's store covers 32
-// consecutive rows of one column, 64 contiguous bytes).
+// forms  v = acc0 + s·acc1  or  v = 16·acc0 - 15·acc1  mod m.  After a slab
+// that is not the last it writes the centred residue back into the
+// accumulators (tcgen05.st) for the next slab to accumulate on; after the
+// last it stores the centred residue as int16, column-major (each thread
+// owns one row; a warp's store covers 32 consecutive rows of one column, 64
+// contiguous bytes).
 //
 // Pipeline: a stage is one (A plane, B plane) pair of 128-byte-deep tiles
 // (32 KiB per CTA), six stages.  Warp 0 of each CTA issues its CTA's TMA
@@ -88,10 +90,6 @@ __device__ __forceinline__ float combine_residue_short(float a0, float a1, bool 
 }
 // int16 encoding of an integer-valued float in [-2^15, 2^15).
 __device__ __forceinline__ uint32_t as_i16_bits(float r) { return __float_as_uint(r + kRoundMagic) & 0xFFFFu; }
-__device__ __forceinline__ float i16_to_float(uint32_t bits16) {
-  return __uint_as_float(0x4B400000u + static_cast<uint32_t>(static_cast<int>(static_cast<int16_t>(bits16)))) -
-         kRoundMagic;
-}
 
 struct EpiCtx {
   int16_t* res;   // r × (m×n column-major, ld = ldr ≥ m; matrix i at i·n·ldr)
@@ -234,7 +232,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           tc_fence_after();
           const int64_t kb1 = min(ksteps, kb0 + slab);
           for (int64_t kb = kb0; kb < kb1 && ok; ++kb) {
-            const uint32_t first = kb == kb0 ? 0u : 1u;
+            const uint32_t first = kb == 0 ? 0u : 1u;  // later slabs add to the carried residue
             if (np == 2) {  // square: stages (d0,e0) and (d1,e1)
               uint32_t s1 = st, p1 = ph;
               next(s1, p1);
@@ -325,6 +323,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           break;
         }
         tc_fence_after();
+        // A slab other than the last leaves its centred residue r in the
+        // accumulators and the next slab accumulates on top of it: acc0 = r,
+        // acc1 = 0 for square moduli (v = acc0 + s·acc1), and acc0 = acc1 = r
+        // for nonsquare ones (16r - 15r = r).  The bounds of Eq. accum-exact
+        // keep their margin: 32768·256 + 544 and 4096·4095 + 255 < 2^24.
+        const bool carry = MODE == 0 && kb0 + slab < ksteps;
         for (int c = 0; c < 64; c += 16) {
           uint32_t v0[16], v1[16];
           tmem_ld16(lane_addr + c, v0);
@@ -333,11 +337,21 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           if (MODE == 1) {
 #pragma unroll
             for (int j = 0; j < 16; ++j) rowmax = fmaxf(rowmax, __uint_as_float(v0[j]));
+          } else if (carry) {  // every lane: tcgen05.st is warp-collective
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+              const float rj =
+                  combine_residue(__uint_as_float(v0[j]), __uint_as_float(v1[j]), square, sb, mf, inv, hi, 0.f);
+              v0[j] = __float_as_uint(rj);
+              v1[j] = square ? 0u : v0[j];
+            }
+            tmem_st16(lane_addr + c, v0);
+            tmem_st16(lane_addr + kAccCols + c, v1);
           } else if (row < ctx.m) {
             const int64_t cc = col0 + c;
             int16_t* dst = rrow + cc * ctx.ldr;
             const int ncol = ctx.n - cc < 16 ? static_cast<int>(ctx.n - cc) : 16;
-            if (ncol == 16 && !kb0 && short_slab) {
+            if (ncol == 16 && short_slab) {  // a single short slab
 #pragma unroll
               for (int j = 0; j < 16; ++j) {
                 const float rj =
@@ -345,7 +359,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
                 *dst = static_cast<int16_t>(as_i16_bits(rj));
                 dst += ctx.ldr;
               }
-            } else if (ncol == 16 && !kb0) {  // the common case: a full chunk, first slab
+            } else if (ncol == 16) {  // the common case: a full chunk
 #pragma unroll
               for (int j = 0; j < 16; ++j) {
                 const float rj =
@@ -354,19 +368,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
                 dst += ctx.ldr;
               }
             } else {
-              float prev[16];
-#pragma unroll
-              for (int j = 0; j < 16; ++j)
-                prev[j] = (kb0 && j < ncol) ? i16_to_float(static_cast<uint16_t>(dst[j * ctx.ldr])) : 0.f;
 #pragma unroll
               for (int j = 0; j < 16; ++j) {
-                const float rj = combine_residue(__uint_as_float(v0[j]), __uint_as_float(v1[j]), square, sb, mf, inv,
-                                                 hi, prev[j]);
+                const float rj =
+                    combine_residue(__uint_as_float(v0[j]), __uint_as_float(v1[j]), square, sb, mf, inv, hi, 0.f);
                 if (j < ncol) dst[j * ctx.ldr] = static_cast<int16_t>(as_i16_bits(rj));
               }
             }
           }
         }
+        if (carry) tmem_st_wait();
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive_remote(acc_empty_leader);

@@ -84,12 +84,15 @@ __global__ void scan_b_kernel(int64_t n, int64_t k, const double* __restrict__ B
 // and the final exponent (0 for rows that are zero in the emulation).
 constexpr int kExpBins = 2112;   // frexp exponents of finite doubles: [-1073, 1024]
 constexpr int kExpBias = 1080;
+constexpr int kFinalizeThreads = 1024;
+constexpr int kBinsPerThread = (kExpBins + kFinalizeThreads - 1) / kFinalizeThreads;
 
-__global__ void finalize_flags_kernel(int64_t m, int64_t n, int* __restrict__ ra,
+__global__ void __launch_bounds__(kFinalizeThreads) finalize_flags_kernel(int64_t m, int64_t n, int* __restrict__ ra,
                                       int* __restrict__ cb, uint8_t* __restrict__ row_flag,
                                       uint8_t* __restrict__ col_flag, unsigned flags,
                                       Oz2Device* dev) {
   __shared__ int hist[kExpBins];
+  __shared__ int warp_sum[32];
   __shared__ int med_s;
   __shared__ int count_s;
   const bool is_a = blockIdx.x == 0;
@@ -104,23 +107,52 @@ __global__ void finalize_flags_kernel(int64_t m, int64_t n, int* __restrict__ ra
     if (kv > 0 && kv < (1 << 20)) atomicAdd(&hist[kv - 2048 + kExpBias], 1);
   }
   __syncthreads();
-  if (threadIdx.x == 0) {
-    int total = 0;
-    for (int b = 0; b < kExpBins; ++b) total += hist[b];
-    int med = 0;
+  // Lower median of the histogram: each thread sums kBinsPerThread bins, a
+  // block-wide inclusive scan of those sums locates the bin that holds the
+  // element of rank ⌊(total-1)/2⌋.
+  {
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    const int b0 = threadIdx.x * kBinsPerThread;
+    int mine = 0;
+#pragma unroll
+    for (int j = 0; j < kBinsPerThread; ++j) mine += b0 + j < kExpBins ? hist[b0 + j] : 0;
+    int incl = mine;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += v;
+    }
+    if (lane == 31) warp_sum[wid] = incl;
+    __syncthreads();
+    if (wid == 0) {
+      int w = lane < kFinalizeThreads / 32 ? warp_sum[lane] : 0;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int v = __shfl_up_sync(0xffffffffu, w, o);
+        if (lane >= o) w += v;
+      }
+      warp_sum[lane] = w;  // inclusive prefix over warps
+    }
+    __syncthreads();
+    incl += wid ? warp_sum[wid - 1] : 0;
+    const int total = warp_sum[kFinalizeThreads / 32 - 1];
+    if (threadIdx.x == 0) med_s = 0;
+    __syncthreads();
     if (total > 0) {
-      int rank = (total - 1) / 2, acc = 0;
-      for (int b = 0; b < kExpBins; ++b) {
-        acc += hist[b];
-        if (acc > rank) {
-          med = b - kExpBias;
-          break;
+      const int rank = (total - 1) / 2;
+      int acc = incl - mine;  // exclusive prefix
+      if (acc <= rank && rank < incl) {
+        for (int j = 0; j < kBinsPerThread; ++j) {
+          acc += hist[b0 + j];
+          if (acc > rank) {
+            med_s = b0 + j - kExpBias;
+            break;
+          }
         }
       }
     }
-    med_s = med;
+    __syncthreads();
   }
-  __syncthreads();
   const int med = med_s;
   const bool window = (flags & OZ2_FLAG_NO_FALLBACK) == 0;
   int local = 0;
@@ -175,7 +207,7 @@ cudaError_t launch_scan(int64_t m, int64_t n, int64_t k, const double* A, int64_
     }
   }
   count_launch();
-  finalize_flags_kernel<<<2, 1024, 0, st>>>(m, n, out.ra, out.cb, out.row_flag, out.col_flag,
+  finalize_flags_kernel<<<2, kFinalizeThreads, 0, st>>>(m, n, out.ra, out.cb, out.row_flag, out.col_flag,
                                             flags, dev);
   return cudaGetLastError();
 }
