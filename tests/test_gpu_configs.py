@@ -7,7 +7,8 @@ span several 256-wide tiles.
 * k = 40000 (the tall-K case: two K-slabs for the square moduli, ten for the
   merged nonsquare ones);
 * k = 64 with φ = 4 and 1% of A's rows scaled by 2^±300 (the wide case:
-  native-FP64 fallback rows).
+  native-FP64 fallback rows);
+* a batched GEMV, Y = A·X with 16 right-hand sides.
 """
 import numpy as np
 import pytest
@@ -83,3 +84,12 @@ def test_k64_wide_character_with_fallback_rows(oz):
     res = orc.evaluate_rows(prep, A, B, rows=rows)
     got = run(oz, A, B, w.r)
     check(got, res, rows)
+
+
+def test_gemv_batch16_character(oz):
+    w = wl.WORKLOADS["gemv_batch16"]
+    A, B = wl.make_inputs(w, m=1500, k=2100)
+    res = orc.oz2_dgemm(A, B, w.r)
+    got = run(oz, A, B, w.r)
+    check(got, res)
+    assert cref.scaled_error(got["C"], A, B, rows=np.arange(0, 1500, 97)) <= 1e-15

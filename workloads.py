@@ -34,7 +34,7 @@ class Workload:
 # The five dense shapes: a small case the oracle finishes in seconds, the
 # square 4096 case, the square 16384 ceiling case, a tall-K case stressing
 # K-chunking, and a k = 64 case with a wide dynamic range and 1% of A's rows
-# scaled by 2^±300 (native-FP64 fallback rows).
+# scaled by 2^±300 (native-FP64 fallback rows); and a batched-GEMV shape.
 WORKLOADS = {
     "dgemm_256": Workload("dgemm_256", 256, 256, 256, 0.5, 12, index=1),
     "dgemm_4096": Workload("dgemm_4096", 4096, 4096, 4096, 0.5, 12, index=2),
@@ -42,6 +42,9 @@ WORKLOADS = {
     "dgemm_tallk": Workload("dgemm_tallk", 1024, 1024, 65536, 0.5, 12, index=4),
     "dgemm_k64_wide": Workload("dgemm_k64_wide", 16384, 16384, 64, 4.0, 12,
                                scaled_rows=0.01, index=5),
+    # Batched GEMV (§3 "Strategy 1"): Y = A·X with a batch of 16 right-hand
+    # sides, through the same kernels.
+    "gemv_batch16": Workload("gemv_batch16", 16384, 16, 16384, 0.5, 12, index=6),
 }
 
 
