@@ -93,8 +93,9 @@ typedef struct {
  * ------------------------------------------------------------------- */
 
 /* C = A·B (overwrite, β = 0) by Ozaki Scheme II with TZ quantiser and R2
- * scales.  Allocates its workspace with cudaMallocAsync on `stream` and
- * frees it on the same stream.  m == 0 or n == 0: no-op; k == 0: C = 0. */
+ * scales.  Allocates its workspace stream-ordered on `stream` from the
+ * library's memory pool (see oz2_trim_memory) and frees it on the same
+ * stream.  m == 0 or n == 0: no-op; k == 0: C = 0. */
 int oz2_dgemm(int64_t m, int64_t n, int64_t k,
               const double* d_A, int64_t lda,
               const double* d_B, int64_t ldb,
@@ -104,7 +105,9 @@ int oz2_dgemm(int64_t m, int64_t n, int64_t k,
 /* As oz2_dgemm with A, B and C in HOST memory (pinned memory gives the
  * best transfer rate).  Copies A and B to the device, computes, copies C
  * back, and synchronises `stream` before returning.  Device buffers and the
- * workspace are allocated and freed stream-ordered inside the call. */
+ * workspace are allocated and freed stream-ordered inside the call, from the
+ * library's memory pool.  A contiguous matrix (ld = rows) moves in one
+ * linear copy, any other in a pitched copy. */
 int oz2_dgemm_host(int64_t m, int64_t n, int64_t k,
                    const double* h_A, int64_t lda,
                    const double* h_B, int64_t ldb,
@@ -185,6 +188,13 @@ int oz2_plane_layout(int num_moduli, int32_t* plane_offset);
 /* Statistics of the last call on the current device (synchronises; resets
  * the timing accumulators and the launch counter). */
 int oz2_get_stats(oz2_stats* out);
+
+/* oz2_dgemm, oz2_dgemm_host and oz2_fallback take their workspace and
+ * staging buffers from a stream-ordered memory pool that the library owns on
+ * each device and that keeps freed blocks for the next call.  This returns
+ * the current device's unused blocks to the system (synchronises the
+ * device).  OZ2_ERR_CUDA on a CUDA failure. */
+int oz2_trim_memory(void);
 
 /* Synchronises the device and returns the device status word (OZ2_OK or
  * OZ2_ERR_TIMEOUT), clearing it. */

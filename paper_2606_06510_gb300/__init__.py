@@ -60,6 +60,7 @@ _SIGS = {
     "oz2_workspace_layout": (_I, [_I64, _I64, _I64, _I, ctypes.POINTER(oz2_ws_layout)]),
     "oz2_plane_layout": (_I, [_I, _P]),
     "oz2_get_stats": (_I, [ctypes.POINTER(oz2_stats)]),
+    "oz2_trim_memory": (_I, []),
     "oz2_check_device_status": (_I, []),
     "oz2_status_string": (ctypes.c_char_p, [_I]),
     "oz2_scan": (_I, [_I64, _I64, _I64, _P, _I64, _P, _I64, _U, _P, _P, _P, _P, _P]),
@@ -199,6 +200,10 @@ def oz2_dgemm_ex(A, B, C=None, num_moduli=12, quant="tz", scale="r2", flags=0, w
                               QUANT[quant], SCALE[scale], flags, _ptr(workspace), workspace.numel(),
                               _stream(stream)), "oz2_dgemm_ex")
     return C, workspace
+
+
+def oz2_trim_memory():
+    _check(lib().oz2_trim_memory(), "oz2_trim_memory")
 
 
 def oz2_get_stats() -> dict:

@@ -217,6 +217,10 @@ struct DeviceState {
   uint32_t* table_a = nullptr;
   uint32_t* table_b = nullptr;
   Oz2Device* status = nullptr;
+  // Stream-ordered pool for the workspaces and staging buffers the library
+  // allocates itself; it keeps freed blocks for reuse (release threshold:
+  // unlimited) until oz2_trim_memory.
+  cudaMemPool_t pool = nullptr;
 };
 static DeviceState g_devs[64];
 static std::mutex g_mu;
@@ -283,10 +287,40 @@ static int device_state(DeviceState** out) {
       return OZ2_ERR_CUDA;
     s.table_a = tables;
     s.table_b = tables + kTableMax;
+    cudaMemPoolProps props;
+    std::memset(&props, 0, sizeof(props));
+    props.allocType = cudaMemAllocationTypePinned;
+    props.location.type = cudaMemLocationTypeDevice;
+    props.location.id = dev;
+    if (cudaMemPoolCreate(&s.pool, &props) == cudaSuccess) {
+      cuuint64_t keep = ~cuuint64_t(0);
+      cudaMemPoolSetAttribute(s.pool, cudaMemPoolAttrReleaseThreshold, &keep);
+    } else {
+      cudaGetLastError();
+      s.pool = nullptr;  // the device's default pool serves instead
+    }
     s.ready = true;
   }
   *out = &s;
   return OZ2_OK;
+}
+
+// Stream-ordered allocation from the library's pool on the current device.
+static cudaError_t pool_alloc(void** p, size_t bytes, cudaStream_t s) {
+  DeviceState* ds = nullptr;
+  if (device_state(&ds) != OZ2_OK) return cudaErrorInitializationError;
+  return ds->pool ? cudaMallocFromPoolAsync(p, bytes, ds->pool, s) : cudaMallocAsync(p, bytes, s);
+}
+
+// Column-major rows × cols matrix copy; one linear copy when both sides are
+// contiguous (ld = rows), a pitched copy otherwise.
+static cudaError_t copy_matrix(double* dst, int64_t dld, const double* src, int64_t sld, int64_t rows, int64_t cols,
+                               cudaMemcpyKind kind, cudaStream_t s) {
+  if (rows == 0 || cols == 0) return cudaSuccess;
+  if ((dld == rows && sld == rows) || cols == 1)
+    return cudaMemcpyAsync(dst, src, sizeof(double) * rows * cols, kind, s);
+  return cudaMemcpy2DAsync(dst, sizeof(double) * dld, src, sizeof(double) * sld, sizeof(double) * rows, cols, kind,
+                           s);
 }
 
 __global__ void reset_status_kernel(Oz2Device* dev) {
@@ -487,7 +521,7 @@ int oz2_dgemm(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, con
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   size_t bytes = oz2_workspace_size(m, n, k, num_moduli);
   void* ws = nullptr;
-  if (cudaMallocAsync(&ws, bytes, s) != cudaSuccess) {
+  if (pool_alloc(&ws, bytes, s) != cudaSuccess) {
     cudaGetLastError();
     return OZ2_ERR_ALLOC;
   }
@@ -509,7 +543,7 @@ int oz2_dgemm_host(int64_t m, int64_t n, int64_t k, const double* hA, int64_t ld
                bC = align256(sizeof(double) * m * n);
   const size_t ws = k > 0 ? oz2_workspace_size(m, n, k, num_moduli) : 0;
   uint8_t* buf = nullptr;
-  if (cudaMallocAsync(reinterpret_cast<void**>(&buf), bA + bB + bC + ws, s) != cudaSuccess) {
+  if (pool_alloc(reinterpret_cast<void**>(&buf), bA + bB + bC + ws, s) != cudaSuccess) {
     cudaGetLastError();
     return OZ2_ERR_ALLOC;
   }
@@ -518,22 +552,27 @@ int oz2_dgemm_host(int64_t m, int64_t n, int64_t k, const double* hA, int64_t ld
   double* dC = reinterpret_cast<double*>(buf + bA + bB);
   cudaError_t err = cudaSuccess;
   if (k > 0) {
-    err = cudaMemcpy2DAsync(dA, sizeof(double) * m, hA, sizeof(double) * lda, sizeof(double) * m, k,
-                            cudaMemcpyHostToDevice, s);
-    if (err == cudaSuccess)
-      err = cudaMemcpy2DAsync(dB, sizeof(double) * k, hB, sizeof(double) * ldb, sizeof(double) * k, n,
-                              cudaMemcpyHostToDevice, s);
+    err = copy_matrix(dA, m, hA, lda, m, k, cudaMemcpyHostToDevice, s);
+    if (err == cudaSuccess) err = copy_matrix(dB, k, hB, ldb, k, n, cudaMemcpyHostToDevice, s);
   }
   if (err == cudaSuccess)
     st = oz2_dgemm_ex(m, n, k, dA, m, dB, std::max<int64_t>(1, k), dC, m, num_moduli, OZ2_QUANT_TZ, OZ2_SCALE_R2,
                       0, k > 0 ? buf + bA + bB + bC : nullptr, ws, stream);
   if (err == cudaSuccess && st == OZ2_OK)
-    err = cudaMemcpy2DAsync(hC, sizeof(double) * ldc, dC, sizeof(double) * m, sizeof(double) * m, n,
-                            cudaMemcpyDeviceToHost, s);
+    err = copy_matrix(hC, ldc, dC, m, m, n, cudaMemcpyDeviceToHost, s);
   cudaFreeAsync(buf, s);
   if (cudaStreamSynchronize(s) != cudaSuccess && err == cudaSuccess) err = cudaErrorUnknown;
   if (st != OZ2_OK) return st;
   return to_status(err);
+}
+
+int oz2_trim_memory(void) {
+  DeviceState* ds = nullptr;
+  const int st = device_state(&ds);
+  if (st) return st;
+  if (cudaDeviceSynchronize() != cudaSuccess) return OZ2_ERR_CUDA;
+  if (ds->pool && cudaMemPoolTrimTo(ds->pool, 0) != cudaSuccess) return OZ2_ERR_CUDA;
+  return OZ2_OK;
 }
 
 int oz2_get_stats(oz2_stats* out) {
@@ -691,7 +730,7 @@ int oz2_fallback(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, 
   if (!row_flag || !col_flag || !C || (k && (!A || !B))) return OZ2_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   int* scratch = nullptr;
-  if (cudaMallocAsync(reinterpret_cast<void**>(&scratch), sizeof(int) * (m + n + 2), s) != cudaSuccess) {
+  if (pool_alloc(reinterpret_cast<void**>(&scratch), sizeof(int) * (m + n + 2), s) != cudaSuccess) {
     cudaGetLastError();
     return OZ2_ERR_ALLOC;
   }
