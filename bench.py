@@ -41,8 +41,8 @@ GEMM_SOURCE = os.path.join(ROOT, "paper_2606_06510_gb300", "csrc", "k_gemm.cu")
 # DRAM read+write bytes of one residue-GEMM launch, from the ncu capture in
 # profiles/residue_gemm_dgemm_4096.md; reported only while the kernel source
 # is the one the counters were taken on.
-GEMM_TRAFFIC = {"workload": "dgemm_4096", "num_moduli": 12, "bytes": 2.1397e9,
-                "sha256": "4686c717ea905cd07908ce0dc16fc747e3b498ba227be082acad73aa7bfddc33"}
+GEMM_TRAFFIC = {"workload": "dgemm_4096", "num_moduli": 12, "bytes": 2.0283e9,
+                "sha256": "1cbdc45098e4a9b8947664cade89443a1272dc0fb90fc094577226f7363b91ae"}
 
 
 def gemm_traffic(w, r):
