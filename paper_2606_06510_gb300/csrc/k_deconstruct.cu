@@ -86,6 +86,24 @@ __device__ __forceinline__ uint32_t e4m3_pow2(int q) {
   return q >= -6 ? static_cast<uint32_t>((q + 7) << 3) : (1u << (q + 9));
 }
 
+// Magnitude-plane code of x: 0 for x = 0, else the E4M3 code of
+// 2^max(-c, ⌈log2|x|⌉ - ex).  A normal double has ⌈log2|x|⌉ = E - 1023, plus
+// one when its fraction is nonzero, read off the high word; subnormals take
+// the general path.
+__device__ __forceinline__ uint32_t magnitude_code(double x, int ex, int c) {
+  const unsigned long long b = __double_as_longlong(x);
+  const uint32_t hi = static_cast<uint32_t>(b >> 32), lo = static_cast<uint32_t>(b);
+  const int E = static_cast<int>((hi >> 20) & 0x7FFu);
+  const bool frac = ((hi & 0xFFFFFu) | lo) != 0;
+  if (E == 0x7FF) return 0u;  // non-finite entries only occur in rows zeroed by the flags
+  if (E == 0) {
+    if (!frac) return 0u;
+    const Split sp = split_double(x);
+    return e4m3_pow2(max(-c, ceil_log2_abs(sp) - ex));
+  }
+  return e4m3_pow2(max(-c, E - 1023 + (frac ? 1 : 0) - ex));
+}
+
 // Gather byte `b` of four 32-bit words into one word (byte 0 from w0 ...).
 __device__ __forceinline__ uint32_t gather_byte(uint32_t w0, uint32_t w1, uint32_t w2, uint32_t w3,
                                                 int b) {
@@ -194,10 +212,7 @@ __global__ void __launch_bounds__(kDecThreads) planes_kernel(OperandView X0, Ope
     if (MODE == 0) {
       uint32_t code[kElems];
 #pragma unroll
-      for (int e = 0; e < kElems; ++e) {
-        const Split sp = split_double(x[e]);
-        code[e] = sp.M ? e4m3_pow2(max(-clamp_c, ceil_log2_abs(sp) - ex)) : 0u;
-      }
+      for (int e = 0; e < kElems; ++e) code[e] = magnitude_code(x[e], ex, clamp_c);
       *reinterpret_cast<uint2*>(dst) = make_uint2(code[0] | (code[1] << 8) | (code[2] << 16) | (code[3] << 24),
                                                   code[4] | (code[5] << 8) | (code[6] << 16) | (code[7] << 24));
     } else {
