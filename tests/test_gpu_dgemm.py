@@ -143,3 +143,33 @@ def test_bench_workload_full_size_sampled(oz):
     assert np.array_equal(v["d"], res.d) and np.array_equal(v["e"], res.e)
     assert_same(C[rows], res.C)
     assert cref.scaled_error(C, A, B, rows=rows[:3]) <= 1e-15
+
+
+def test_cuda_graph_capture_and_replay(oz):
+    """The production calls are stream-ordered end to end (pool allocation,
+    memsets, launches), so they can be captured into a CUDA graph; replays
+    on new input values in the same buffers give the direct call's bits."""
+    import torch
+    A1, B1 = wl.make_inputs(wl.WORKLOADS["dgemm_256"], m=300, n=200, k=333)
+    A2, B2 = wl.random_matrix(300, 333, 1.0, 77), wl.random_matrix(333, 200, 1.0, 78)
+    dA, dB = to_dev(A1), to_dev(B1)
+    C = torch.empty((200, 300), dtype=torch.float64, device="cuda").t()
+    ws = torch.empty(oz.oz2_workspace_size(300, 200, 333, 12), dtype=torch.uint8, device="cuda")
+    s = torch.cuda.Stream()
+    for call in ("dgemm", "dgemm_ex"):
+        run = (lambda: oz.oz2_dgemm(dA, dB, C=C, num_moduli=12, stream=s)) if call == "dgemm" else \
+              (lambda: oz.oz2_dgemm_ex(dA, dB, C=C, num_moduli=12, workspace=ws, stream=s))
+        with torch.cuda.stream(s):
+            run()                                   # warm-up outside the capture (device set-up)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=s):
+            run()
+        for A, B in ((A2, B2), (A1, B1)):
+            dA.copy_(to_dev(A))
+            dB.copy_(to_dev(B))
+            g.replay()
+            torch.cuda.synchronize()
+            want = oz.oz2_dgemm(to_dev(A), to_dev(B), num_moduli=12).cpu().numpy()
+            assert_same(C.cpu().numpy(), want)
+        assert oz.oz2_check_device_status() == 0
