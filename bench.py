@@ -259,7 +259,7 @@ def run_oz2(args):
     achieved = gemm_flops / (gemm_ms * 1e-3) / 1e12
     roofline = {"bound": "tensor", "achieved": round(achieved, 1), "peak": round(fp8_peak, 1), "unit": "TFLOP/s",
                 "frac": round(achieved / fp8_peak, 4), "traffic": gemm_traffic(w, r),
-                "kernel": "plane_gemm_tc_kernel<0> (residue GEMM, 3r FP8 plane products)",
+                "kernel": "plane_gemm_kernel<0> (residue GEMM, 3r FP8 plane products)",
                 "peak_source": f"{pk['source']} bf16 {regime} x {FP8_TO_BF16} (nominal FP8/BF16 ratio); "
                                f"SM clock in the timed region {clk.get('sm_mhz')} of {clk.get('sm_max_mhz')} MHz",
                 "frac_of_nominal_fp8": round(achieved / NOMINAL_FP8_TFLOPS, 4),
@@ -305,11 +305,23 @@ def run_oz2(args):
         extra["native_fp64"] = {"ms": round(native_ms, 3), "TFLOPS": round(w.flops / (native_ms * 1e-3) / 1e12, 3),
                                 "kernel": "fma_gemm_kernel (FP64 FMA chains, 64x64 tiles)"}
         if not args.no_sweep:
-            sweep = {}
+            sweep, speed = {}, {}
             for rr in range(6, 15):
                 Cr = oz.oz2_dgemm(dA, dB, num_moduli=rr)
                 sweep[str(rr)] = float(f"{cref.scaled_error(Cr.cpu().numpy(), A, B, rows=rows[:2]):.3e}")
+                wsr = torch.empty(oz.oz2_workspace_size(w.m, w.n, w.k, rr), dtype=torch.uint8, device=dev)
+                for _ in range(3):
+                    oz.oz2_dgemm_ex(dA, dB, C=dC, num_moduli=rr, workspace=wsr)
+                r0, r1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                r0.record(stream)
+                for _ in range(10):
+                    oz.oz2_dgemm_ex(dA, dB, C=dC, num_moduli=rr, workspace=wsr)
+                r1.record(stream)
+                torch.cuda.synchronize()
+                speed[str(rr)] = round(w.flops / (r0.elapsed_time(r1) / 10 * 1e-3) / 1e12, 2)
+                del wsr
             extra["error_vs_r"] = sweep
+            extra["tflops_vs_r"] = speed
         if world == 1 and not args.no_cpu_baseline:
             extra["cpu_baseline"] = cpu_baseline(w, r, A, B)
 
