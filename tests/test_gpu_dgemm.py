@@ -173,3 +173,48 @@ def test_cuda_graph_capture_and_replay(oz):
             want = oz.oz2_dgemm(to_dev(A), to_dev(B), num_moduli=12).cpu().numpy()
             assert_same(C.cpu().numpy(), want)
         assert oz.oz2_check_device_status() == 0
+
+
+@pytest.mark.parametrize("pad", [(3, 5, 7), (1, 0, 2), (8, 8, 8)])
+def test_leading_dimensions_larger_than_rows(oz, pad):
+    """A, B and C as sub-matrix views of larger column-major arrays (lda > m,
+    ldb > k, ldc > m, odd and even paddings): the same bits as contiguous
+    operands, and C's padding rows are left untouched."""
+    import torch
+    m, n, k = 261, 133, 299
+    A, B = wl.make_inputs(wl.WORKLOADS["dgemm_256"], m=m, n=n, k=k)
+    res = orc.oz2_dgemm(A, B, 12)
+    pa, pb, pc = pad
+    bigA = torch.full((k, m + pa), 7.0, dtype=torch.float64, device="cuda")
+    bigB = torch.full((n, k + pb), -3.0, dtype=torch.float64, device="cuda")
+    bigC = torch.full((n, m + pc), 11.0, dtype=torch.float64, device="cuda")
+    dA = bigA.t()[:m, :]
+    dB = bigB.t()[:k, :]
+    dC = bigC.t()[:m, :]
+    dA.copy_(torch.from_numpy(np.ascontiguousarray(A)).cuda())
+    dB.copy_(torch.from_numpy(np.ascontiguousarray(B)).cuda())
+    assert dA.stride() == (1, m + pa) and dB.stride() == (1, k + pb) and dC.stride() == (1, m + pc)
+    oz.oz2_dgemm(dA, dB, C=dC, num_moduli=12)
+    assert_same(dC.cpu().numpy(), res.C)
+    if pc:
+        assert (bigC.t()[m:, :] == 11.0).all()
+    assert oz.oz2_check_device_status() == 0
+
+
+def test_concurrent_calls_on_two_streams(oz):
+    """Two different problems issued back to back on two streams (each call
+    with its own workspace from the library pool) give their own results."""
+    import torch
+    A1, B1 = wl.make_inputs(wl.WORKLOADS["dgemm_256"], m=300, n=270, k=260)
+    A2, B2 = wl.random_matrix(200, 500, 1.0, 91), wl.random_matrix(500, 180, 1.0, 92)
+    want1, want2 = orc.oz2_dgemm(A1, B1, 12).C, orc.oz2_dgemm(A2, B2, 13).C
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+    d = [to_dev(x) for x in (A1, B1, A2, B2)]
+    torch.cuda.synchronize()
+    for _ in range(3):
+        C1 = oz.oz2_dgemm(d[0], d[1], num_moduli=12, stream=s1)
+        C2 = oz.oz2_dgemm(d[2], d[3], num_moduli=13, stream=s2)
+        torch.cuda.synchronize()
+        assert_same(C1.cpu().numpy(), want1)
+        assert_same(C2.cpu().numpy(), want2)
+    assert oz.oz2_check_device_status() == 0
