@@ -189,6 +189,15 @@ int oz2_plane_layout(int num_moduli, int32_t* plane_offset);
  * the timing accumulators and the launch counter). */
 int oz2_get_stats(oz2_stats* out);
 
+/* Self-test of the failure path.  Launches one warp that waits on an
+ * mbarrier nothing arrives at, bounded by limit_cycles SM cycles (1000 to
+ * 4e9), and on expiry records OZ2_ERR_TIMEOUT in the device status word, as
+ * every library kernel does when one of its waits expires.  The wait ends by
+ * its bound: nothing faults or hangs.  The next oz2_check_device_status then
+ * returns OZ2_ERR_TIMEOUT and clears the word.  OZ2_ERR_INVALID_ARG for a
+ * limit out of range. */
+int oz2_selftest_timeout(long long limit_cycles, void* stream);
+
 /* oz2_dgemm, oz2_dgemm_host and oz2_fallback take their workspace and
  * staging buffers from a stream-ordered memory pool that the library owns on
  * each device and that keeps freed blocks for the next call.  This returns

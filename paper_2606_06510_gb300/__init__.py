@@ -61,6 +61,7 @@ _SIGS = {
     "oz2_plane_layout": (_I, [_I, _P]),
     "oz2_get_stats": (_I, [ctypes.POINTER(oz2_stats)]),
     "oz2_trim_memory": (_I, []),
+    "oz2_selftest_timeout": (_I, [ctypes.c_longlong, _P]),
     "oz2_check_device_status": (_I, []),
     "oz2_status_string": (ctypes.c_char_p, [_I]),
     "oz2_scan": (_I, [_I64, _I64, _I64, _P, _I64, _P, _I64, _U, _P, _P, _P, _P, _P]),
@@ -200,6 +201,10 @@ def oz2_dgemm_ex(A, B, C=None, num_moduli=12, quant="tz", scale="r2", flags=0, w
                               QUANT[quant], SCALE[scale], flags, _ptr(workspace), workspace.numel(),
                               _stream(stream)), "oz2_dgemm_ex")
     return C, workspace
+
+
+def oz2_selftest_timeout(limit_cycles: int = 2_000_000, stream=None):
+    _check(lib().oz2_selftest_timeout(limit_cycles, _stream(stream)), "oz2_selftest_timeout")
 
 
 def oz2_trim_memory():

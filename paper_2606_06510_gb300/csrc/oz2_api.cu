@@ -613,6 +613,33 @@ int oz2_get_stats(oz2_stats* out) {
   return OZ2_OK;
 }
 
+namespace oz2 {
+// One warp waits on an mbarrier that nothing arrives at, bounded by `limit`
+// SM cycles, and on expiry records the timeout as every library kernel does.
+__global__ void timeout_probe_kernel(Oz2Device* dev, long long limit) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x == 0) {
+    const uint32_t b = smem_u32(&bar);
+    mbar_init(b, 1);
+    fence_barrier_init();
+    if (!mbar_wait_bounded(b, 0, limit)) {
+      dev->status = kStatusTimeout;
+      dev->timeout_site = 9;
+    }
+  }
+}
+}  // namespace oz2
+
+int oz2_selftest_timeout(long long limit_cycles, void* stream) {
+  if (limit_cycles < 1000 || limit_cycles > 4000000000LL) return OZ2_ERR_INVALID_ARG;
+  DeviceState* ds = nullptr;
+  const int st = device_state(&ds);
+  if (st) return st;
+  count_launch();
+  timeout_probe_kernel<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(ds->status, limit_cycles);
+  return to_status(cudaGetLastError());
+}
+
 int oz2_check_device_status(void) {
   DeviceState* ds = nullptr;
   int st = device_state(&ds);

@@ -17,7 +17,7 @@ def oz():
 
 def test_every_header_symbol_is_exported(oz):
     names = header_functions()
-    assert len(names) == 19
+    assert len(names) == 20
     raw = ctypes.CDLL(oz.LIB_PATH)
     missing = [n for n in names if not hasattr(raw, n)]
     assert not missing
@@ -50,6 +50,8 @@ def test_host_argument_errors(oz):
     assert L.oz2_dgemm_ex(8, 8, 8, 1, 8, 1, 8, 1, 8, 12, 5, 0, 0, null, 0, null) == -1
     assert L.oz2_dgemm_ex(8, 8, 8, 1, 8, 1, 8, 1, 8, 12, 0, 0, 0, null, 0, null) == -3
     assert L.oz2_dgemm_ex(8, 8, 8, 1, 8, 1, 8, 1, 8, 12, 0, 0, 0, 3, 1 << 30, null) == -3
+    # failure-path self-test: limit out of range
+    assert L.oz2_selftest_timeout(10, null) == -1
     # stage entries: residue leading dimension below m
     assert L.oz2_residue_gemm(8, 8, 8, 12, 1, 1, 1, 7, null) == -1
     assert L.oz2_reconstruct(8, 8, 12, 1, 7, 1, 1, 1, 8, null) == -1

@@ -218,3 +218,19 @@ def test_concurrent_calls_on_two_streams(oz):
         assert_same(C1.cpu().numpy(), want1)
         assert_same(C2.cpu().numpy(), want2)
     assert oz.oz2_check_device_status() == 0
+
+
+def test_wait_expiry_is_reported_and_the_context_stays_usable(oz):
+    """The failure path of every bounded wait, without a GPU fault: a wait
+    that nothing completes expires after ~1 ms, the host reads
+    OZ2_ERR_TIMEOUT once, and the next emulated DGEMM is exact."""
+    import torch
+    assert oz.oz2_check_device_status() == 0
+    oz.oz2_selftest_timeout(2_000_000)
+    torch.cuda.synchronize()
+    assert oz.oz2_check_device_status() == -5         # OZ2_ERR_TIMEOUT
+    assert oz.oz2_check_device_status() == 0          # read once, then cleared
+    A, B = wl.make_inputs(wl.WORKLOADS["dgemm_256"], m=130, n=70, k=90)
+    C = oz.oz2_dgemm(to_dev(A), to_dev(B), num_moduli=12).cpu().numpy()
+    assert_same(C, orc.oz2_dgemm(A, B, 12).C)
+    assert oz.oz2_check_device_status() == 0
