@@ -6,20 +6,30 @@
 // Tiled CUDA-core DGEMM over index lists: 64×64 output tiles, 256 threads,
 // 4×4 outputs per thread, k staged through shared memory in chunks of 16.
 // The same kernel is the cuBLAS-free native comparator (identity lists).
+#include <algorithm>
+
 #include "oz2_common.cuh"
 
 namespace oz2 {
 
 constexpr int kFT = 64, kFK = 16;
 
-// Compact the indices whose flag has bit0 set into `list`, counting in *count.
-__global__ void compact_flags_kernel(int64_t cnt, const uint8_t* __restrict__ flag, int* __restrict__ list,
-                                     int* __restrict__ count) {
-  int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  if (i < cnt && (flag[i] & 1)) list[atomicAdd(count, 1)] = static_cast<int>(i);
+// Compact the rows (blockIdx.y = 0) and columns (blockIdx.y = 1) whose flag
+// has bit0 set into their lists, counting in count[0] and count[1].
+__global__ void compact_flags_kernel(int64_t m, int64_t n, const uint8_t* __restrict__ row_flag,
+                                     const uint8_t* __restrict__ col_flag, int* __restrict__ row_list,
+                                     int* __restrict__ col_list, int* __restrict__ count) {
+  const bool cols = blockIdx.y == 1;
+  const int64_t cnt = cols ? n : m;
+  const uint8_t* flag = cols ? col_flag : row_flag;
+  int* list = cols ? col_list : row_list;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < cnt; i += (int64_t)gridDim.x * blockDim.x)
+    if (flag[i] & 1) list[atomicAdd(count + (cols ? 1 : 0), 1)] = static_cast<int>(i);
 }
 
-// rows: row_list ? row_list[0..*row_count) : 0..m-1 ; cols likewise.
+// rows: row_list ? row_list[0..*row_count) : 0..m-1 ; cols likewise.  With
+// gridDim.y = 2 the blocks with blockIdx.y = 0 take the row list against all
+// columns and those with blockIdx.y = 1 all rows against the column list.
 __global__ void __launch_bounds__(256) fma_gemm_kernel(int64_t m, int64_t n, int64_t k,
                                                        const double* __restrict__ A, int64_t lda,
                                                        const double* __restrict__ B, int64_t ldb,
@@ -31,6 +41,13 @@ __global__ void __launch_bounds__(256) fma_gemm_kernel(int64_t m, int64_t n, int
   __shared__ double As[kFK][kFT + 1];
   __shared__ double Bs[kFK][kFT + 1];
   __shared__ int rid[kFT], cid[kFT];
+  if (gridDim.y == 2) {
+    if (blockIdx.y == 0) {
+      col_list = nullptr;
+    } else {
+      row_list = nullptr;
+    }
+  }
   const int64_t nr = row_list ? *row_count : m;
   const int64_t nc = col_list ? *col_count : n;
   const int64_t rt = (nr + kFT - 1) / kFT, ct = (nc + kFT - 1) / kFT;
@@ -99,23 +116,26 @@ static int fb_grid() {
   return sms * 4;
 }
 
-// scratch: (m + n + 2) ints of device memory (lists and counts).
+// scratch: (m + n + 2) ints of device memory (counts, then the lists); the
+// two counts must be zero on entry unless `zero_counts` is set.
 cudaError_t launch_fallback_lists(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, const double* B,
                                   int64_t ldb, const uint8_t* row_flag, const uint8_t* col_flag, int* scratch,
-                                  double* C, int64_t ldc, cudaStream_t st) {
+                                  double* C, int64_t ldc, cudaStream_t st, bool zero_counts) {
   if (m == 0 || n == 0) return cudaSuccess;
   int* counts = scratch;              // [0]: rows, [1]: cols
   int* rlist = scratch + 2;
   int* clist = rlist + m;
-  cudaError_t err = cudaMemsetAsync(counts, 0, 2 * sizeof(int), st);
-  if (err != cudaSuccess) return err;
-  count_launch(4);
-  compact_flags_kernel<<<static_cast<unsigned>((m + 255) / 256), 256, 0, st>>>(m, row_flag, rlist, counts);
-  compact_flags_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, st>>>(n, col_flag, clist, counts + 1);
-  const int g = fb_grid();
-  // flagged rows × all columns, then all rows × flagged columns
-  fma_gemm_kernel<<<g, 256, 0, st>>>(m, n, k, A, lda, B, ldb, rlist, counts, nullptr, nullptr, C, ldc);
-  fma_gemm_kernel<<<g, 256, 0, st>>>(m, n, k, A, lda, B, ldb, nullptr, nullptr, clist, counts + 1, C, ldc);
+  if (zero_counts) {
+    const cudaError_t err = cudaMemsetAsync(counts, 0, 2 * sizeof(int), st);
+    if (err != cudaSuccess) return err;
+  }
+  count_launch(2);
+  const int64_t most = m > n ? m : n;
+  const unsigned cg = static_cast<unsigned>(std::min<int64_t>((most + 255) / 256, 4096));
+  compact_flags_kernel<<<dim3(cg, 2), 256, 0, st>>>(m, n, row_flag, col_flag, rlist, clist, counts);
+  // flagged rows × all columns (blockIdx.y = 0), all rows × flagged columns (1)
+  fma_gemm_kernel<<<dim3(fb_grid(), 2), 256, 0, st>>>(m, n, k, A, lda, B, ldb, rlist, counts, clist, counts + 1, C,
+                                                       ldc);
   return cudaGetLastError();
 }
 

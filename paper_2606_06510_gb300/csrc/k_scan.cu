@@ -177,10 +177,11 @@ __global__ void __launch_bounds__(kFinalizeThreads) finalize_flags_kernel(int64_
 
 cudaError_t launch_scan(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda,
                         const double* B, int64_t ldb, unsigned flags, ScanOut out,
-                        Oz2Device* dev, cudaStream_t st) {
+                        Oz2Device* dev, cudaStream_t st, bool zero_keys) {
   cudaError_t err;
-  if (m > 0 && (err = cudaMemsetAsync(out.ra, 0, sizeof(int) * m, st)) != cudaSuccess) return err;
-  if (n > 0 && (err = cudaMemsetAsync(out.cb, 0, sizeof(int) * n, st)) != cudaSuccess) return err;
+  // The scan keys are maxima taken with atomics: zero unless the caller has.
+  if (zero_keys && m > 0 && (err = cudaMemsetAsync(out.ra, 0, sizeof(int) * m, st)) != cudaSuccess) return err;
+  if (zero_keys && n > 0 && (err = cudaMemsetAsync(out.cb, 0, sizeof(int) * n, st)) != cudaSuccess) return err;
   if (k > 0) {
     int chunk = 64;
     int64_t ks = (k + chunk - 1) / chunk;

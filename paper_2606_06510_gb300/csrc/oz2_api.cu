@@ -330,6 +330,29 @@ __global__ void reset_status_kernel(Oz2Device* dev) {
   dev->s = 0;
 }
 
+// The start of a call: the status summary, and the workspace words that
+// later stages accumulate with atomics (scan keys ra, cb; the "+1" row
+// maxima; the two fallback counts) set to zero, in one launch.
+__global__ void prepare_call_kernel(Oz2Device* dev, int* ra, int64_t m, int* cb, int64_t n, float* urow,
+                                    int* counts) {
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    dev->fallback_rows = 0;
+    dev->fallback_cols = 0;
+    dev->u_max_bits = 0;
+    dev->s = 0;
+    counts[0] = 0;
+    counts[1] = 0;
+  }
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < m + n; i += (int64_t)gridDim.x * blockDim.x) {
+    if (i < m) {
+      ra[i] = 0;
+      urow[i] = 0.f;
+    } else {
+      cb[i - m] = 0;
+    }
+  }
+}
+
 void count_launch(int n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
 
 static size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
@@ -475,13 +498,16 @@ int oz2_dgemm_ex(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, 
 
   cudaError_t err = cudaSuccess;
   count_launch();
-  reset_status_kernel<<<1, 1, 0, s>>>(ds->status);
+  {
+    const int64_t blocks = std::min<int64_t>((m + n + 255) / 256, 1024);
+    prepare_call_kernel<<<static_cast<unsigned>(std::max<int64_t>(blocks, 1)), 256, 0, s>>>(ds->status, ra, m, cb,
+                                                                                              n, urow, misc);
+  }
   mark(0);
   if (err == cudaSuccess)
-    err = launch_scan(m, n, k, A, lda, B, ldb, flags, ScanOut{ra, cb, rf, cf}, ds->status, s);
+    err = launch_scan(m, n, k, A, lda, B, ldb, flags, ScanOut{ra, cb, rf, cf}, ds->status, s, false);
   mark(1);
   if (scale == OZ2_SCALE_R2) {
-    if (err == cudaSuccess) err = cudaMemsetAsync(urow, 0, sizeof(float) * m, s);
     if (err == cudaSuccess)
       err = launch_magnitude_planes(m, n, k, A, lda, B, ldb, ra, cb, rf, cf, mag_a, mag_b, s);
     mark(2);
@@ -502,7 +528,7 @@ int oz2_dgemm_ex(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, 
   mark(6);
   if (err == cudaSuccess) err = launch_reconstruct(m, n, mods, res, L.res_ld, d, e, C, ldc, s);
   mark(7);
-  if (err == cudaSuccess) err = launch_fallback_lists(m, n, k, A, lda, B, ldb, rf, cf, misc, C, ldc, s);
+  if (err == cudaSuccess) err = launch_fallback_lists(m, n, k, A, lda, B, ldb, rf, cf, misc, C, ldc, s, false);
   mark(8);
 
   hs.k_slab = static_cast<int>(std::min<int64_t>(kKSlabMerged, L.k_pad));
@@ -667,7 +693,8 @@ int oz2_scan(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, cons
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   count_launch();
   reset_status_kernel<<<1, 1, 0, s>>>(ds->status);
-  return to_status(launch_scan(m, n, k, A, lda, B, ldb, flags, ScanOut{ra, cb, row_flag, col_flag}, ds->status, s));
+  return to_status(
+      launch_scan(m, n, k, A, lda, B, ldb, flags, ScanOut{ra, cb, row_flag, col_flag}, ds->status, s, true));
 }
 
 int oz2_scale(int64_t m, int64_t n, int64_t k, int num_moduli, const double* A, int64_t lda, const double* B,
@@ -761,7 +788,7 @@ int oz2_fallback(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, 
     cudaGetLastError();
     return OZ2_ERR_ALLOC;
   }
-  cudaError_t err = launch_fallback_lists(m, n, k, A, lda, B, ldb, row_flag, col_flag, scratch, C, ldc, s);
+  cudaError_t err = launch_fallback_lists(m, n, k, A, lda, B, ldb, row_flag, col_flag, scratch, C, ldc, s, true);
   cudaFreeAsync(scratch, s);
   return to_status(err);
 }

@@ -382,7 +382,7 @@ struct ScanOut {
 };
 cudaError_t launch_scan(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda,
                         const double* B, int64_t ldb, unsigned flags, ScanOut out,
-                        Oz2Device* dev, cudaStream_t st);
+                        Oz2Device* dev, cudaStream_t st, bool zero_keys);
 cudaError_t launch_magnitude_planes(int64_t m, int64_t n, int64_t k, const double* A,
                                     int64_t lda, const double* B, int64_t ldb, const int32_t* ra,
                                     const int32_t* cb, const uint8_t* row_flag,
@@ -408,7 +408,7 @@ cudaError_t launch_reconstruct(int64_t m, int64_t n, const Oz2Moduli& mods,
 cudaError_t launch_fallback_lists(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda,
                                   const double* B, int64_t ldb, const uint8_t* row_flag,
                                   const uint8_t* col_flag, int* scratch, double* C, int64_t ldc,
-                                  cudaStream_t st);
+                                  cudaStream_t st, bool zero_counts);
 cudaError_t launch_native(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda,
                           const double* B, int64_t ldb, double* C, int64_t ldc, cudaStream_t st);
 }  // namespace oz2
