@@ -234,3 +234,43 @@ def test_wait_expiry_is_reported_and_the_context_stays_usable(oz):
     C = oz.oz2_dgemm(to_dev(A), to_dev(B), num_moduli=12).cpu().numpy()
     assert_same(C, orc.oz2_dgemm(A, B, 12).C)
     assert oz.oz2_check_device_status() == 0
+
+
+@pytest.mark.parametrize("seed", range(12))
+def test_randomised_problems_bit_exact(oz, seed):
+    """Seeded random problems: shapes 1..300, exponent spread φ ∈ [0, 6],
+    r ∈ [1, 16], every quantiser/scale variant, and planted special rows and
+    columns (zeros, 2^±300 scaling, subnormal entries, an Inf or NaN).  Every
+    entry of C, d and e bit-exact against the oracle."""
+    rng = np.random.default_rng(4000 + seed)
+    m, n, k = (int(v) for v in rng.integers(1, 301, size=3))
+    phi = float(rng.uniform(0.0, 6.0))
+    r = int(rng.integers(1, 17))
+    quant = ("tz", "rn")[seed % 2]
+    scale = ("r2", "r1")[(seed // 2) % 2] if seed % 3 else "r2"
+    A = np.array(wl.random_matrix(m, k, phi, 5000 + seed), order="F")
+    B = np.array(wl.random_matrix(k, n, phi, 6000 + seed), order="F")
+    for _ in range(int(rng.integers(0, 4))):           # planted rows of A
+        i, kind = int(rng.integers(0, m)), int(rng.integers(0, 5))
+        if kind == 0:
+            A[i, :] = 0.0
+        elif kind == 1:
+            A[i, :] *= 2.0 ** 300
+        elif kind == 2:
+            A[i, :] *= 2.0 ** -300
+        elif kind == 3:
+            A[i, int(rng.integers(0, k))] = 5e-324 * int(rng.integers(1, 1000))
+        else:
+            A[i, int(rng.integers(0, k))] = (np.inf, -np.inf, np.nan)[int(rng.integers(0, 3))]
+    for _ in range(int(rng.integers(0, 3))):           # planted columns of B
+        j, kind = int(rng.integers(0, n)), int(rng.integers(0, 3))
+        if kind == 0:
+            B[:, j] = 0.0
+        elif kind == 1:
+            B[:, j] *= 2.0 ** -200
+        else:
+            B[int(rng.integers(0, k)), j] = np.nan
+    res = orc.oz2_dgemm(A, B, r, quant=quant, scale=scale)
+    C, v = run_ex(oz, A, B, r, quant=quant, scale=scale)
+    assert np.array_equal(v["d"], res.d) and np.array_equal(v["e"], res.e)
+    assert_same(C, res.C)
