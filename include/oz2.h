@@ -155,7 +155,8 @@ int oz2_dgemm_ex(int64_t m, int64_t n, int64_t k,
  *   row_flag[m], col_flag[n] uint8  bit0 fallback, bit1 zero in emulation
  *   d[m], e[n]            int32  the scale exponents (D = diag 2^d_i ...)
  *   urow[m]               float  max_j U_ij of the "+1" GEMM (R2)
- *   mag_a, mag_b          uint8  magnitude planes Â (m×k_pad), B̂ (n×k_pad)
+ *   mag_a, mag_b          uint8  magnitude planes Â (m×k_pad), B̂ (n×k_pad),
+ *                                row-major
  *   planes_a, planes_b    uint8  E4M3 digit planes, see oz2_plane_layout
  *   residues              int16  r matrices C^(i), each m×n column-major
  *                                with ld = res_ld (matrix i starts at element
@@ -173,9 +174,16 @@ int oz2_workspace_layout(int64_t m, int64_t n, int64_t k, int num_moduli,
                          oz2_ws_layout* out);
 
 /* Digit-plane layout (§2.5).  For operand X with `rows` rows (m for A, n
- * for B) every plane is a rows×k_pad byte matrix, row-major (k contiguous),
- * zero-padded from k to k_pad; plane p starts at byte p·rows·k_pad.  The
- * planes of modulus i are consecutive, starting at plane_offset[i]:
+ * for B) there are P planes (the return value), each logically a rows×k_pad
+ * byte matrix zero-padded from k to k_pad, stored as 128 × 128-byte blocks
+ * with the rows padded to rows_pad = ⌈rows/128⌉·128 (pad rows hold zero
+ * digits): byte l of row `row` of plane p is at
+ *   ((⌊row/128⌋·(k_pad/128) + ⌊l/128⌋)·P + p)·16384 + (row mod 128)·128
+ *     + (l mod 128),
+ * so a plane buffer holds P·rows_pad·k_pad bytes, each block is one MMA
+ * operand tile, and the P blocks of one (row block, k-block) are
+ * consecutive.  The planes of modulus i are consecutive, starting at
+ * plane_offset[i]:
  *   square m_i = s²:  (d0, d1)              d = d0 + s·d1, balanced base s
  *   nonsquare, B:     (d0+d1, d0, d1)       d = d0 + 16·d1, carry-corrected
  *   nonsquare, A:     (d0+d1, d0, -16·d1)   (pre-scaled for the merged
@@ -239,7 +247,7 @@ int oz2_scale(int64_t m, int64_t n, int64_t k, int num_moduli,
 
 /* Stage 3 (Eq. scale and Algorithm 1 "lin:dec"): Ã = ⌊2^d_i A_il⌉ and
  * B̃ = ⌊2^e_j B_lj⌉, their centred residues, and the E4M3 digit planes in
- * the oz2_plane_layout order.  Rows with row_flag bit1 (columns with
+ * the layout of oz2_plane_layout.  Rows with row_flag bit1 (columns with
  * col_flag bit1) are written as zero. */
 int oz2_deconstruct(int64_t m, int64_t n, int64_t k, int num_moduli,
                     const double* d_A, int64_t lda, const double* d_B, int64_t ldb,
@@ -249,7 +257,7 @@ int oz2_deconstruct(int64_t m, int64_t n, int64_t k, int num_moduli,
                     void* stream);
 
 /* Stage 4 (Eq. modgemm, Eq. sq-shortcut, Eq. kar): from digit planes in
- * the oz2_plane_layout order (k_pad = k rounded up to 128), the residue
+ * the layout of oz2_plane_layout (k_pad = k rounded up to 128), the residue
  * matrices C^(i) = (A^(i) B^(i)) mod m_i, centred, as r int16 matrices,
  * each m×n column-major with leading dimension ldr ≥ m (matrix i starts at
  * element i·n·ldr; rows m..ldr-1 are not written).  Three FP8 tcgen05 MMAs

@@ -257,13 +257,19 @@ def oz2_scale(A, B, ra, cb, rf, cf, num_moduli=12, quant="tz", scale="r2", strea
     return mag_a, mag_b, urow, d, e
 
 
+def plane_storage_shape(rows: int, k_pad: int, num_planes: int) -> tuple:
+    """Shape of the digit-plane storage of an operand with `rows` rows:
+    (row blocks, k-blocks, planes, 128 rows, 128 bytes), rows padded to 128."""
+    return ((rows + 127) // 128, k_pad // 128, num_planes, 128, 128)
+
+
 def oz2_deconstruct(A, B, d, e, rf, cf, num_moduli=12, quant="tz", stream=None):
     m, k = A.shape
     n = B.shape[1]
     k_pad = (k + 127) // 128 * 128
     _, P = oz2_plane_layout(num_moduli)
-    pa = torch.empty((P, m, k_pad), dtype=torch.uint8, device=A.device)
-    pb = torch.empty((P, n, k_pad), dtype=torch.uint8, device=A.device)
+    pa = torch.empty(plane_storage_shape(m, k_pad, P), dtype=torch.uint8, device=A.device)
+    pb = torch.empty(plane_storage_shape(n, k_pad, P), dtype=torch.uint8, device=A.device)
     _check(lib().oz2_deconstruct(m, n, k, num_moduli, _ptr(A), _ld(A), _ptr(B), _ld(B), _ptr(d), _ptr(e), _ptr(rf),
                                  _ptr(cf), QUANT[quant], _ptr(pa), _ptr(pb), _stream(stream)), "oz2_deconstruct")
     return pa, pb
@@ -275,7 +281,8 @@ def residue_ld(m: int) -> int:
 
 
 def oz2_residue_gemm(planes_a, planes_b, m, n, k, num_moduli=12, simt=False, stream=None):
-    """planes: uint8 CUDA tensors (P, rows, k_pad).  Returns an int16 view of
+    """planes: uint8 CUDA tensors in the storage layout oz2_deconstruct returns
+    (plane_storage_shape).  Returns an int16 view of
     shape (r, m, n) over column-major storage (r, n, ldr), ldr = residue_ld(m)."""
     ldr = residue_ld(m)
     res = torch.empty((num_moduli, n, ldr), dtype=torch.int16, device=planes_a.device)
@@ -344,8 +351,10 @@ def workspace_views(ws: torch.Tensor, m: int, n: int, k: int, num_moduli: int) -
         "urow": view(L["urow"], m, torch.float32, (m,)),
         "mag_a": view(L["mag_a"], m * k_pad, torch.uint8, (m, k_pad)),
         "mag_b": view(L["mag_b"], n * k_pad, torch.uint8, (n, k_pad)),
-        "planes_a": view(L["planes_a"], P * m * k_pad, torch.uint8, (P, m, k_pad)),
-        "planes_b": view(L["planes_b"], P * n * k_pad, torch.uint8, (P, n, k_pad)),
+        "planes_a": view(L["planes_a"], P * ((m + 127) // 128 * 128) * k_pad, torch.uint8,
+                         plane_storage_shape(m, k_pad, P)),
+        "planes_b": view(L["planes_b"], P * ((n + 127) // 128 * 128) * k_pad, torch.uint8,
+                         plane_storage_shape(n, k_pad, P)),
         "residues": view(L["residues"], num_moduli * n * L["res_ld"], torch.int16,
                          (num_moduli, n, L["res_ld"]))[:, :, :m].transpose(1, 2),
     }

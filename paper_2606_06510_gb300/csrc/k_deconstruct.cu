@@ -20,17 +20,22 @@
 namespace oz2 {
 
 constexpr int kElems = 8;  // k-entries per thread
-constexpr int kDecThreads = 256;
 
-// Tile shape of each pass: threads per row, k-entries per tile column (a
-// divisor of the k padding) and rows per block.
+// Launch and tile shape of each pass: threads per block, resident blocks per
+// SM (64 registers a thread either way), threads per row, k-entries per tile
+// column (a divisor of the k padding) and rows per block.  The
+// deconstruction's blocks are large so that two of them, each with its own
+// copy of the digit-plane table, fill an SM.
 template <int MODE>
 struct TileShape {
+  static constexpr int kThreads = MODE == 0 ? 256 : 512;
+  static constexpr int kBlocksPerSm = MODE == 0 ? 8 : 2;
   static constexpr int kThreadsPerRow = MODE == 0 ? 4 : 16;
   static constexpr int kSeg = kElems * kThreadsPerRow;
-  static constexpr int kRows = kDecThreads / kThreadsPerRow;
+  static constexpr int kRows = kThreads / kThreadsPerRow;
 };
 static_assert(kKPad % TileShape<0>::kSeg == 0 && kKPad % TileShape<1>::kSeg == 0, "tile column must divide k_pad");
+static_assert(TileShape<1>::kSeg == kPlaneLine, "a row's threads write whole plane lines");
 
 // Integer significand M and exponent x with |x| = M·2^x (M < 2^53), or M = 0.
 struct Split {
@@ -104,6 +109,13 @@ __device__ __forceinline__ uint32_t magnitude_code(double x, int ex, int c) {
   return e4m3_pow2(max(-c, E - 1023 + (frac ? 1 : 0) - ex));
 }
 
+// Rows a pass writes: the magnitude plane has the operand's rows, the digit
+// planes whole 128-row blocks.
+template <int MODE>
+__host__ __device__ __forceinline__ int64_t rows_stored(int64_t rows) {
+  return MODE == 0 ? rows : (rows + kPlaneRows - 1) / kPlaneRows * kPlaneRows;
+}
+
 // Gather byte `b` of four 32-bit words into one word (byte 0 from w0 ...).
 __device__ __forceinline__ uint32_t gather_byte(uint32_t w0, uint32_t w1, uint32_t w2, uint32_t w3,
                                                 int b) {
@@ -143,39 +155,49 @@ __device__ __forceinline__ void load8(const OperandView& X, int64_t row, int64_t
 
 // Residues of 8 entries modulo modulus I and their E4M3 digit planes (the
 // modulus's constants are compile-time constants).
+//
+// Ã = u0 + u1·2^16 + u2·2^32 + u3·2^48 with u3 signed (|Ã| < 2^62, so
+// |u3| ≤ 2^14), and b = 4·(u0 + kDecBias).  Then
+//   Y = b + 4·(u1·(2^16 mod m) + u2·(2^32 mod m) + u3·(2^48 mod m))
+// is 4·y with y ≡ Ã + kDecBias (mod m) and 2^24 < y < 2^28 (the bias
+// outweighs the most negative u3 term).  With magic = ⌈2^30/m⌉,
+// q = ⌊Y·magic/2^32⌋ = ⌊y/m + y·(magic·m - 2^30)/(m·2^30)⌋ is ⌊y/m⌋ or one
+// more, since the second term is below y/2^30 < 1; so Y - 4qm = 4(y - qm) is
+// the byte offset of the entry for y mod m in a table whose 2m entries
+// start m entries before it.  The table is rotated by kDecBias.
 template <int I>
-__device__ __forceinline__ void planes_one(const uint32_t (&u0)[kElems], const uint32_t (&u1)[kElems],
-                                           const uint32_t (&u2)[kElems], const uint32_t (&u3)[kElems],
-                                           const uint32_t (&ng)[kElems], const uint32_t* table, uint8_t* dst,
-                                           size_t plane_stride) {
+__device__ __forceinline__ void planes_one(const uint32_t (&b)[kElems], const uint32_t (&u1)[kElems],
+                                           const uint32_t (&u2)[kElems], const int (&u3)[kElems],
+                                           const uint32_t* table, uint8_t* dst) {
   constexpr ModConst mc = mod_const(I);
+  const char* centre = reinterpret_cast<const char*>(table + mc.table_off + mc.m);
   uint32_t w[kElems];
 #pragma unroll
   for (int e = 0; e < kElems; ++e) {
-    // Ã mod m from the limbs: u0 + u1·2^16 + u2·2^32 + u3·2^48 - ng·2^64 (mod m), < 2^28
-    const uint32_t y = u0[e] + u1[e] * mc.limb1 + u2[e] * mc.limb2 + u3[e] * mc.limb3 + ng[e] * mc.neg64;
-    w[e] = table[mc.table_off + mod_magic(y, mc.m, mc.magic, mc.sh)];  // packed E4M3 planes of centred(r)
+    const uint32_t Y = b[e] + u1[e] * mc.limb1 + u2[e] * mc.limb2 + static_cast<uint32_t>(u3[e]) * mc.limb3;
+    const uint32_t q = __umulhi(Y, mc.magic);
+    const int off = static_cast<int>(Y - q * static_cast<uint32_t>(4 * mc.m));  // in [-4m, 4m)
+    w[e] = *reinterpret_cast<const uint32_t*>(centre + off);  // packed E4M3 planes of centred(Ã mod m)
   }
-  uint8_t* pdst = dst + static_cast<size_t>(mc.plane_off) * plane_stride;
+  uint8_t* pdst = dst + mc.plane_off * kPlaneBlock;
 #pragma unroll
   for (int p = 0; p < (mc.s ? 2 : 3); ++p)
-    *reinterpret_cast<uint2*>(pdst + p * plane_stride) =
+    *reinterpret_cast<uint2*>(pdst + p * kPlaneBlock) =
         make_uint2(gather_byte(w[0], w[1], w[2], w[3], p), gather_byte(w[4], w[5], w[6], w[7], p));
 }
 
 template <int... Is>
-__device__ __forceinline__ void planes_all(std::integer_sequence<int, Is...>, const uint32_t (&u0)[kElems],
+__device__ __forceinline__ void planes_all(std::integer_sequence<int, Is...>, const uint32_t (&b)[kElems],
                                            const uint32_t (&u1)[kElems], const uint32_t (&u2)[kElems],
-                                           const uint32_t (&u3)[kElems], const uint32_t (&ng)[kElems],
-                                           const uint32_t* table, uint8_t* dst, size_t plane_stride) {
-  (planes_one<Is>(u0, u1, u2, u3, ng, table, dst, plane_stride), ...);
+                                           const int (&u3)[kElems], const uint32_t* table, uint8_t* dst) {
+  (planes_one<Is>(b, u1, u2, u3, table, dst), ...);
 }
 
 // MODE 0: magnitude plane (1 plane); MODE 1: residue digit planes for the
 // first R moduli (R is a template parameter so the modulus loop unrolls and
 // every per-modulus constant and plane offset is known at compile time).
 template <int MODE, int R>
-__global__ void __launch_bounds__(kDecThreads) planes_kernel(OperandView X0, OperandView X1, int blocks0, int64_t k,
+__global__ void __launch_bounds__(TileShape<MODE>::kThreads, TileShape<MODE>::kBlocksPerSm) planes_kernel(OperandView X0, OperandView X1, int blocks0, int64_t k,
                                                              int64_t k_pad, int clamp_c, int rn,
                                                              const __grid_constant__ Oz2Moduli mods) {
   extern __shared__ uint32_t table[];
@@ -188,22 +210,34 @@ __global__ void __launch_bounds__(kDecThreads) planes_kernel(OperandView X0, Ope
     __syncthreads();
   }
   using TS = TileShape<MODE>;
-  const int64_t row_tiles = (X.rows + TS::kRows - 1) / TS::kRows;
+  const int64_t rows_out = rows_stored<MODE>(X.rows);
+  const int64_t row_tiles = (rows_out + TS::kRows - 1) / TS::kRows;
   const int64_t ntiles = row_tiles * (k_pad / TS::kSeg);
   const int part = threadIdx.x & (TS::kThreadsPerRow - 1);
   const int rloc = threadIdx.x / TS::kThreadsPerRow;
-  const size_t plane_stride = static_cast<size_t>(X.rows) * k_pad;
 
   for (int64_t tile = bid; tile < ntiles; tile += nblocks) {
     const int64_t kt = tile / row_tiles;  // consecutive blocks share a k-slice of many rows
     const int64_t row = (tile - kt * row_tiles) * TS::kRows + rloc;
-    if (row >= X.rows) continue;
+    if (row >= rows_out) continue;
     const int64_t l0 = kt * TS::kSeg + part * kElems;
+    const bool pad = row >= X.rows;  // pad rows of the last block: zero digits
     double x[kElems];
-    load8(X, row, l0, k, x);  // entries of rows zeroed by the flags are replaced below
-    const bool zero_row = (X.flag[row] & 2) != 0;
-    const int ex = X.exps[row];
-    uint8_t* dst = X.out + static_cast<size_t>(row) * k_pad + l0;
+    if (pad) {
+#pragma unroll
+      for (int e = 0; e < kElems; ++e) x[e] = 0.0;
+    } else {
+      load8(X, row, l0, k, x);  // entries of rows zeroed by the flags are replaced below
+    }
+    const bool zero_row = pad || (X.flag[row] & 2) != 0;
+    const int ex = pad ? 0 : X.exps[row];
+    // Magnitude plane: row-major rows × k_pad.  Digit planes: 128 × 128-byte
+    // blocks, those of one (row block, k-block) consecutive.
+    uint8_t* dst =
+        MODE == 0 ? X.out + static_cast<size_t>(row) * k_pad + l0
+                  : X.out + ((static_cast<size_t>(row / kPlaneRows) * (k_pad / kPlaneLine) + l0 / kPlaneLine) *
+                                 num_planes(R) * kPlaneBlock +
+                             (row % kPlaneRows) * kPlaneLine + l0 % kPlaneLine);
     if (zero_row) {
 #pragma unroll
       for (int e = 0; e < kElems; ++e) x[e] = 0.0;
@@ -216,24 +250,23 @@ __global__ void __launch_bounds__(kDecThreads) planes_kernel(OperandView X0, Ope
       *reinterpret_cast<uint2*>(dst) = make_uint2(code[0] | (code[1] << 8) | (code[2] << 16) | (code[3] << 24),
                                                   code[4] | (code[5] << 8) | (code[6] << 16) | (code[7] << 24));
     } else {
-      // Quantise (Eq. scale) and split Ã, as a 64-bit two's complement word,
-      // into 16-bit limbs; the sign enters the residue as one more term,
-      // neg·((-2^64) mod m).
-      uint32_t u0[kElems], u1[kElems], u2[kElems], u3[kElems], ng[kElems];
+      // Quantise (Eq. scale) and split Ã, a 64-bit two's complement word,
+      // into three unsigned 16-bit limbs and a signed top limb.
+      uint32_t b[kElems], u1[kElems], u2[kElems];
+      int u3[kElems];
 #pragma unroll
       for (int e = 0; e < kElems; ++e) {
         const Split sp = split_double(x[e]);
         const unsigned long long a = quantise_abs(sp, ex, rn != 0);
-        const bool neg = sp.neg && a != 0;
-        const unsigned long long t = neg ? 0ull - a : a;
-        const uint32_t lo = static_cast<uint32_t>(t), hi = static_cast<uint32_t>(t >> 32);
-        u0[e] = lo & 0xFFFFu;
+        const unsigned long long t = sp.neg ? 0ull - a : a;
+        const uint32_t lo = static_cast<uint32_t>(t);
+        const int hi = static_cast<int>(t >> 32);
+        b[e] = ((lo << 2) & 0x3FFFCu) | (4u * kDecBias);
         u1[e] = lo >> 16;
-        u2[e] = hi & 0xFFFFu;
+        u2[e] = static_cast<uint32_t>(hi) & 0xFFFFu;
         u3[e] = hi >> 16;
-        ng[e] = neg ? 1u : 0u;
       }
-      planes_all(std::make_integer_sequence<int, R>{}, u0, u1, u2, u3, ng, table, dst, plane_stride);
+      planes_all(std::make_integer_sequence<int, R>{}, b, u1, u2, u3, table, dst);
     }
   }
 }
@@ -248,7 +281,7 @@ static int num_sms() {
 template <int MODE>
 static int64_t tiles_of(int64_t rows, int64_t k_pad) {
   using TS = TileShape<MODE>;
-  return ((rows + TS::kRows - 1) / TS::kRows) * (k_pad / TS::kSeg);
+  return ((rows_stored<MODE>(rows) + TS::kRows - 1) / TS::kRows) * (k_pad / TS::kSeg);
 }
 
 // Split a grid of about `blocks_per_sm` × SMs blocks between the two operands
@@ -279,11 +312,11 @@ cudaError_t launch_magnitude_planes(int64_t m, int64_t n, int64_t k, const doubl
   OperandView va{A, 1, lda, m, ra, row_flag, mag_a, nullptr, 0};
   OperandView vb{B, ldb, 1, n, cb, col_flag, mag_b, nullptr, vec_ok(B, ldb, 1)};
   int g0, g1;
-  split_grid(m ? tiles_of<0>(m, k_pad) : 0, n ? tiles_of<0>(n, k_pad) : 0, 8, &g0, &g1);
+  split_grid(m ? tiles_of<0>(m, k_pad) : 0, n ? tiles_of<0>(n, k_pad) : 0, TileShape<0>::kBlocksPerSm, &g0, &g1);
   if (g0 + g1 == 0) return cudaSuccess;
   if (g0 == 0) va = vb;
   count_launch();
-  planes_kernel<0, 0><<<g0 + g1, kDecThreads, 0, st>>>(va, vb, g0, k, k_pad, c, 0, dummy);
+  planes_kernel<0, 0><<<g0 + g1, TileShape<0>::kThreads, 0, st>>>(va, vb, g0, k, k_pad, c, 0, dummy);
   return cudaGetLastError();
 }
 
@@ -298,7 +331,7 @@ cudaError_t launch_deconstruct(int64_t m, int64_t n, int64_t k, const Oz2Moduli&
   OperandView va{A, 1, lda, m, d, row_flag, planes_a, table_a, 0};
   OperandView vb{B, ldb, 1, n, e, col_flag, planes_b, table_b, vec_ok(B, ldb, 1)};
   int g0, g1;
-  split_grid(m ? tiles_of<1>(m, k_pad) : 0, n ? tiles_of<1>(n, k_pad) : 0, 4, &g0, &g1);
+  split_grid(m ? tiles_of<1>(m, k_pad) : 0, n ? tiles_of<1>(n, k_pad) : 0, TileShape<1>::kBlocksPerSm, &g0, &g1);
   if (g0 + g1 == 0) return cudaSuccess;
   if (g0 == 0) va = vb;
   cudaError_t err = cudaSuccess;
@@ -309,7 +342,7 @@ cudaError_t launch_deconstruct(int64_t m, int64_t n, int64_t k, const Oz2Moduli&
     err = cudaFuncSetAttribute(planes_kernel<1, R>, cudaFuncAttributeMaxDynamicSharedMemorySize,            \
                                static_cast<int>(smem));                                                     \
     if (err == cudaSuccess)                                                                                 \
-      planes_kernel<1, R><<<g0 + g1, kDecThreads, smem, st>>>(va, vb, g0, k, k_pad, 0, rn, mods);          \
+      planes_kernel<1, R><<<g0 + g1, TileShape<1>::kThreads, smem, st>>>(va, vb, g0, k, k_pad, 0, rn, mods); \
     break;
     OZ2_DEC_CASE(1) OZ2_DEC_CASE(2) OZ2_DEC_CASE(3) OZ2_DEC_CASE(4) OZ2_DEC_CASE(5) OZ2_DEC_CASE(6)
     OZ2_DEC_CASE(7) OZ2_DEC_CASE(8) OZ2_DEC_CASE(9) OZ2_DEC_CASE(10) OZ2_DEC_CASE(11) OZ2_DEC_CASE(12)

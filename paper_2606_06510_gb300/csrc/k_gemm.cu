@@ -180,6 +180,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         const int pbase = MODE == 0 ? mods.plane_off[i] : 0;
         const int ya = static_cast<int>(tm * kTileM + rank * kRows);
         const int yb = static_cast<int>(tn * kTileN + rank * kRows);
+        // Digit planes: first line of block (row block, k-block 0, plane pbase);
+        // successive k-blocks are nplanes blocks apart.  A row block past the
+        // operand's last one lies past the end of the tensor (zero fill).
+        const int64_t blk_a = (static_cast<int64_t>(ya / kPlaneRows) * ksteps * mods.nplanes + pbase) * kPlaneRows;
+        const int64_t blk_b = (static_cast<int64_t>(yb / kPlaneRows) * ksteps * mods.nplanes + pbase) * kPlaneRows;
         for (int64_t kb = 0; kb < ksteps && ok; ++kb) {
           for (int p = 0; p < np; ++p, ++it) {
             const int s = it % kStages;
@@ -189,9 +194,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
             }
             if (leader) mbar_arrive_expect_tx(full0 + 8 * s, 2u * kStageBytes);
             const uint32_t sa = smem_u32(smem + s * kStageBytes);
-            const int x = static_cast<int>(kb * kBK);
-            tma_load_3d_pair(sa, &tmA, full_leader0 + 8 * s, x, ya, pbase + p);
-            tma_load_3d_pair(sa + kTileBytes, &tmB, full_leader0 + 8 * s, x, yb, pbase + p);
+            if (MODE == 0) {
+              const int64_t off = (kb * mods.nplanes + p) * kPlaneRows;
+              tma_load_2d_pair(sa, &tmA, full_leader0 + 8 * s, 0, static_cast<int>(blk_a + off));
+              tma_load_2d_pair(sa + kTileBytes, &tmB, full_leader0 + 8 * s, 0, static_cast<int>(blk_b + off));
+            } else {
+              const int x = static_cast<int>(kb * kBK);
+              tma_load_3d_pair(sa, &tmA, full_leader0 + 8 * s, x, ya, 0);
+              tma_load_3d_pair(sa + kTileBytes, &tmB, full_leader0 + 8 * s, x, yb, 0);
+            }
           }
         }
       }
@@ -418,10 +429,9 @@ __global__ void plane_gemm_simt_kernel(const uint8_t* __restrict__ pa, const uin
   const int64_t row = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   const int64_t col = blockIdx.y;
   if (row >= ctx.m || col >= ctx.n) return;
-  const size_t sa = static_cast<size_t>(ctx.m) * k_pad, sbs = static_cast<size_t>(ctx.n) * k_pad;
   const uint8_t* ar = pa + row * k_pad;
   const uint8_t* bc = pb + col * k_pad;
-  if (MODE == 1) {
+  if (MODE == 1) {  // magnitude planes: one plane, rows × k_pad
     float acc = 0.f;
     for (int64_t l = 0; l < k_pad; ++l) acc += e4m3_to_float(ar[l]) * e4m3_to_float(bc[l]);
     atomicMax(reinterpret_cast<int*>(ctx.urow) + row, __float_as_int(acc));
@@ -433,20 +443,26 @@ __global__ void plane_gemm_simt_kernel(const uint8_t* __restrict__ pa, const uin
     const float mf = static_cast<float>(mods.m[i]);
     const float inv = 1.f / mf;
     const float hi = static_cast<float>(mods.m[i] - 1 - mods.m[i] / 2);
-    const size_t p0 = mods.plane_off[i];
     const int64_t slab = square ? kKSlabSquare : kKSlabMerged;
+    // Byte l of plane plane_off + j of row `rw` (of A) or column (of B), in
+    // 128 × 128-byte blocks.
+    const int64_t kblocks = k_pad / kPlaneLine;
+    auto plane = [&](const uint8_t* base, int64_t rw, int j, int64_t l) {
+      const int64_t blk = ((rw / kPlaneRows) * kblocks + l / kPlaneLine) * mods.nplanes + mods.plane_off[i] + j;
+      return e4m3_to_float(base[blk * kPlaneBlock + (rw % kPlaneRows) * kPlaneLine + l % kPlaneLine]);
+    };
     float res = 0.f;
     for (int64_t l0 = 0; l0 < k_pad; l0 += slab) {
       float a0 = 0.f, a1 = 0.f;
       const int64_t l1 = min(k_pad, l0 + slab);
       for (int64_t l = l0; l < l1; ++l) {
-        const float x0 = e4m3_to_float(ar[p0 * sa + l]), y0 = e4m3_to_float(bc[p0 * sbs + l]);
-        const float x1 = e4m3_to_float(ar[(p0 + 1) * sa + l]), y1 = e4m3_to_float(bc[(p0 + 1) * sbs + l]);
+        const float x0 = plane(pa, row, 0, l), y0 = plane(pb, col, 0, l);
+        const float x1 = plane(pa, row, 1, l), y1 = plane(pb, col, 1, l);
         if (square) {
           a0 += x0 * y0;
           a1 += x1 * y0 + x0 * y1;
         } else {
-          const float x2 = e4m3_to_float(ar[(p0 + 2) * sa + l]), y2 = e4m3_to_float(bc[(p0 + 2) * sbs + l]);
+          const float x2 = plane(pa, row, 2, l), y2 = plane(pb, col, 2, l);
           a0 += x0 * y0;
           a1 += x1 * y1 + x2 * y2;
         }
@@ -477,17 +493,37 @@ static EncodeTiledFn get_encode_fn() {
   return fn;
 }
 
-// Planes of one operand: `np` planes of rows × k_pad bytes, row-major; the
-// box is 128 rows × 128 bytes with the 128-byte swizzle the MMA descriptors use.
-static bool make_plane_map(CUtensorMap* map, const uint8_t* base, int64_t rows, int64_t k_pad, int np) {
+// Magnitude plane of one operand: rows × k_pad bytes, row-major; the box is
+// 128 rows × 128 bytes with the 128-byte swizzle the MMA descriptors use.
+static bool make_plane_map(CUtensorMap* map, const uint8_t* base, int64_t rows, int64_t k_pad) {
   EncodeTiledFn enc = get_encode_fn();
   if (!enc) return false;
-  cuuint64_t dims[3] = {static_cast<cuuint64_t>(k_pad), static_cast<cuuint64_t>(rows),
-                        static_cast<cuuint64_t>(np)};
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(k_pad), static_cast<cuuint64_t>(rows), 1};
   cuuint64_t strides[2] = {static_cast<cuuint64_t>(k_pad), static_cast<cuuint64_t>(rows * k_pad)};
   cuuint32_t box[3] = {kBK, static_cast<cuuint32_t>(kRows), 1};
   cuuint32_t estr[3] = {1, 1, 1};
   CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, const_cast<uint8_t*>(base), dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+// Digit planes of one operand (128 × 128-byte blocks, rows padded to 128) as
+// a 2-D tensor of 128-byte lines; the box is one whole block, which lands in
+// shared memory as the 128-row tile the MMA descriptors expect, with the
+// 128-byte swizzle.  Line coordinates are int32: the planes of one operand
+// stay below 2^38 bytes.
+static bool make_block_map(CUtensorMap* map, const uint8_t* base, int64_t rows, int64_t k_pad, int np) {
+  static_assert(kBK == kPlaneLine && kRows == kPlaneRows, "one MMA operand tile is one plane block");
+  EncodeTiledFn enc = get_encode_fn();
+  if (!enc) return false;
+  const int64_t lines = (rows + kPlaneRows - 1) / kPlaneRows * kPlaneRows * (k_pad / kPlaneLine) * np;
+  if (lines + 2 * static_cast<int64_t>(kPlaneRows) * (k_pad / kPlaneLine) * np > 0x7FFFFFFFLL) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(kPlaneLine), static_cast<cuuint64_t>(lines)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(kPlaneLine)};
+  cuuint32_t box[2] = {kBK, static_cast<cuuint32_t>(kRows)};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t*>(base), dims, strides, box, estr,
                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
@@ -516,10 +552,11 @@ cudaError_t launch_plane_gemm(int64_t m, int64_t n, int64_t k_pad, const Oz2Modu
     else plane_gemm_simt_kernel<1><<<g, 128, 0, st>>>(planes_a, planes_b, mods, k_pad, ctx);
     return cudaGetLastError();
   }
-  const int np = mode == 0 ? mods.nplanes : 1;
   CUtensorMap ta, tb;
-  if (!make_plane_map(&ta, planes_a, m, k_pad, np) || !make_plane_map(&tb, planes_b, n, k_pad, np))
-    return cudaErrorInvalidValue;
+  const bool maps = mode == 0 ? make_block_map(&ta, planes_a, m, k_pad, mods.nplanes) &&
+                                    make_block_map(&tb, planes_b, n, k_pad, mods.nplanes)
+                              : make_plane_map(&ta, planes_a, m, k_pad) && make_plane_map(&tb, planes_b, n, k_pad);
+  if (!maps) return cudaErrorInvalidValue;
   UnitMap um;
   um.ntm = (m + kTileM - 1) / kTileM;
   um.ntn = (n + kTileN - 1) / kTileN;

@@ -16,10 +16,11 @@ namespace oz2 {
 // extension primes used for r = 13..16 (nonsquare, < 513).
 static const int kModuliAll[kMaxModuli] = {1089, 1024, 961, 841, 625, 529, 511, 509,
                                            503,  499,  491, 487, 479, 467, 463, 461};
-constexpr int kTableMax = 10240;  // Σ of all sixteen moduli = 9939 entries
+constexpr int kTableMax = 20480;  // 2·Σ of all sixteen moduli = 19878 entries
 
-// Packed E4M3 digit planes of every residue (byte p = plane p), per modulus;
-// table 0 for A (last nonsquare plane pre-scaled by -16), table 1 for B.
+// Packed E4M3 digit planes of every residue (byte p = plane p), 2m entries
+// per modulus, entry i for the residue (i - kDecBias) mod m; table 0 for A
+// (last nonsquare plane pre-scaled by -16), table 1 for B.
 static __device__ uint32_t g_plane_table[2][kTableMax];
 // Device status block (sticky status word, fallback counts, scale summary).
 static __device__ Oz2Device g_status;
@@ -159,7 +160,7 @@ static Oz2Moduli build_moduli(int r, int quant) {
     c.invp[i] = static_cast<uint32_t>((static_cast<u64>(c.inv[i]) << 32) / static_cast<u64>(m));
   }
   c.nplanes = plane;
-  c.table_entries = toff;
+  c.table_entries = 2 * toff;
   // Direct-CRT constants.
   for (int k = 0; k < r; ++k) {
     const int mk = kModuliAll[k];
@@ -268,13 +269,14 @@ static int device_state(DeviceState** out) {
       int off = 0;
       for (int i = 0; i < kMaxModuli; ++i) {
         const int m = kModuliAll[i];
-        for (int r = 0; r < m; ++r) {
-          int d = r > m - 1 - m / 2 ? r - m : r;  // centred residue
-          uint32_t w = plane_word(d, m, t == 0);
+        for (int j = 0; j < 2 * m; ++j) {
+          const int r = floor_mod(j - kDecBias % m, m);
+          const int d = r > m - 1 - m / 2 ? r - m : r;  // centred residue
+          const uint32_t w = plane_word(d, m, t == 0);
           if (w == 0xFFFFFFFFu) return OZ2_ERR_CUDA;
-          host_table[t][off + r] = w;
+          host_table[t][off + j] = w;
         }
-        off += m;
+        off += 2 * m;
       }
     }
     if (cudaMemcpyToSymbol(g_plane_table, host_table, sizeof(host_table)) != cudaSuccess) return OZ2_ERR_CUDA;
@@ -377,8 +379,9 @@ static void compute_layout(int64_t m, int64_t n, int64_t k, int r, oz2_ws_layout
   L->misc = take(4 * (m + n + 2));
   L->mag_a = take(static_cast<size_t>(m) * k_pad);
   L->mag_b = take(static_cast<size_t>(n) * k_pad);
-  L->planes_a = take(static_cast<size_t>(planes) * m * k_pad);
-  L->planes_b = take(static_cast<size_t>(planes) * n * k_pad);
+  // Digit planes in 128 × 128-byte blocks: rows padded to a multiple of 128.
+  L->planes_a = take(static_cast<size_t>(planes) * ((m + 127) / 128 * 128) * k_pad);
+  L->planes_b = take(static_cast<size_t>(planes) * ((n + 127) / 128 * 128) * k_pad);
   const int64_t res_ld = (m + 7) / 8 * 8;  // 16-byte columns
   L->residues = take(2 * static_cast<size_t>(r) * n * res_ld);
   L->total = off;

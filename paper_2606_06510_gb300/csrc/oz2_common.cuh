@@ -31,15 +31,19 @@ constexpr int kKSlabMerged = 4096;
 constexpr int kModuliList[kMaxModuli] = {1089, 1024, 961, 841, 625, 529, 511, 509,
                                          503,  499,  491, 487, 479, 467, 463, 461};
 
+// The deconstruction's digit-plane table holds 2m entries per modulus
+// (entry i: the planes of the residue (i - kDecBias) mod m), so that a
+// quotient one too large, and the bias that keeps the residue sum positive,
+// cost nothing at the lookup.
+constexpr int kDecBias = 1 << 25;
+
 struct ModConst {
   int m;
   int s;          // square base, 0 for nonsquare moduli
   int plane_off;  // first plane of this modulus
-  int table_off;  // first entry of this modulus in the digit-plane table
-  uint32_t limb1, limb2, limb3;  // 2^16, 2^32, 2^48 mod m
-  uint32_t neg64;                // (-2^64) mod m
-  uint32_t magic;                // ⌈2^(32+sh)/m⌉
-  int sh;                        // ⌊log2(m-1)⌋
+  int table_off;  // first of this modulus's 2m entries in the digit-plane table
+  uint32_t limb1, limb2, limb3;  // 4·(2^16 mod m), 4·(2^32 mod m), 4·(2^48 mod m)
+  uint32_t magic;                // ⌈2^30/m⌉
 };
 
 constexpr int ce_isqrt(int m) {
@@ -47,14 +51,26 @@ constexpr int ce_isqrt(int m) {
   while ((s + 1) * (s + 1) <= m) ++s;
   return s * s == m ? s : 0;
 }
-constexpr int ce_log2_floor(unsigned v) {
-  int r = -1;
-  while (v) {
-    v >>= 1;
-    ++r;
-  }
-  return r;
+// Digit planes of an operand with `rows` rows are stored as 128 × 128-byte
+// blocks: rows are padded to a multiple of 128 (the pad rows hold zero
+// digits), and byte l of row `row` of plane p is at
+//   ((⌊row/128⌋·(k_pad/128) + ⌊l/128⌋)·P + p)·2^14 + (row mod 128)·128 + l mod 128
+// for P planes in all.  One block is exactly the tile the residue GEMM loads
+// for an MMA operand (one contiguous 16 KiB TMA box), and the P blocks of a
+// (row block, k-block) are consecutive, so a thread of the deconstruction
+// reaches the same row segment of every plane at compile-time offsets.
+constexpr int kPlaneLine = 128;                            // bytes of a row segment (k-entries)
+constexpr int kPlaneRows = 128;                            // rows of a block
+constexpr int kPlaneBlock = kPlaneLine * kPlaneRows;       // 16 KiB
+
+// Planes stored for the first r moduli (two per square modulus, three per
+// nonsquare one).
+constexpr int num_planes(int r) {
+  int p = 0;
+  for (int j = 0; j < r; ++j) p += ce_isqrt(kModuliList[j]) ? 2 : 3;
+  return p;
 }
+
 constexpr ModConst mod_const(int i) {
   ModConst c{};
   int plane = 0, toff = 0;
@@ -66,15 +82,12 @@ constexpr ModConst mod_const(int i) {
   c.m = m;
   c.s = ce_isqrt(m);
   c.plane_off = plane;
-  c.table_off = toff;
+  c.table_off = 2 * toff;
   const unsigned long long um = static_cast<unsigned long long>(m);
-  c.limb1 = static_cast<uint32_t>((1ull << 16) % um);
-  c.limb2 = static_cast<uint32_t>((1ull << 32) % um);
-  c.limb3 = static_cast<uint32_t>((1ull << 48) % um);
-  const unsigned long long two64 = ((~0ull) % um + 1) % um;  // 2^64 mod m
-  c.neg64 = static_cast<uint32_t>((um - two64) % um);
-  c.sh = ce_log2_floor(static_cast<unsigned>(m - 1));
-  c.magic = static_cast<uint32_t>(((1ull << (32 + c.sh)) + um - 1) / um);
+  c.limb1 = static_cast<uint32_t>(4 * ((1ull << 16) % um));
+  c.limb2 = static_cast<uint32_t>(4 * ((1ull << 32) % um));
+  c.limb3 = static_cast<uint32_t>(4 * ((1ull << 48) % um));
+  c.magic = static_cast<uint32_t>(((1ull << 30) + um - 1) / um);
   return c;
 }
 
@@ -118,7 +131,7 @@ struct Oz2Moduli {
   int crt_g[kMaxModuli];
   int crt_ml, crt_mlh;
   int crt_m51l, crt_m51h;
-  int table_entries;            // Σ m_i
+  int table_entries;            // 2·Σ m_i (digit-plane table, 2m entries per modulus)
 };
 
 // Per-device status block (in device global memory, owned by oz2_api.cu).
@@ -132,14 +145,6 @@ struct Oz2Device {
   int pad[10];
 };
 
-// Residue of y (< 2^31) modulo m with a precomputed multiplier
-// (Granlund & Montgomery 1994, "Division by invariant integers using
-// multiplication"): q = ⌊y·magic / 2^(32+sh)⌋ = ⌊y/m⌋ because the error
-// e = magic·m - 2^(32+sh) < m and y·e < 2^(32+sh) for y < 2^31.
-__device__ __forceinline__ uint32_t mod_magic(uint32_t y, uint32_t m, uint32_t magic, int sh) {
-  uint32_t q = __umulhi(y, magic) >> sh;
-  return y - q * m;
-}
 
 // ---------------------------------------------------------------------------
 // PTX wrappers (sm_100-family tcgen05 / TMA / mbarrier), with bounded waits.
@@ -227,6 +232,13 @@ __device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr) {
 }
 // 3-D tiled TMA load issued by either CTA of a pair; the transaction bytes
 // complete on `bar` (a shared::cluster address, here the leader CTA's barrier).
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap* map, uint32_t bar, int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cta.global.tile.mbarrier::complete_tx::bytes.cta_group::2"
+      " [%0], [%1, {%3, %4}], [%2];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(x), "r"(y)
+      : "memory");
+}
 __device__ __forceinline__ void tma_load_3d_pair(uint32_t dst, const CUtensorMap* map, uint32_t bar, int x, int y,
                                                  int z) {
   asm volatile(

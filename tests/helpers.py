@@ -32,10 +32,12 @@ def to_dev(x, dtype=None):
 
 
 def planes_from_residues(resid, mods, oz_oracle, k_pad, merged=False):
-    """Oracle digit planes (E4M3 codes) of centred residue matrices, library layout.
+    """Oracle digit planes (E4M3 codes) of centred residue matrices, in the
+    library's storage layout.
 
     resid: list over moduli of (rows, k) int arrays of centred residues.
-    Returns uint8 array (P, rows, k_pad).
+    Returns a uint8 array (⌈rows/128⌉, k_pad/128, P, 128, 128): 128 × 128-byte
+    blocks (row block, k-block, plane, row in block, byte), pad rows zero.
     """
     rows, k = resid[0].shape
     planes = []
@@ -44,4 +46,9 @@ def planes_from_residues(resid, mods, oz_oracle, k_pad, merged=False):
             buf = np.zeros((rows, k_pad), dtype=np.uint8)
             buf[:, :k] = oz_oracle.e4m3_encode_array(p)
             planes.append(buf)
-    return np.stack(planes)
+    P = len(planes)
+    rows_pad = (rows + 127) // 128 * 128
+    full = np.zeros((P, rows_pad, k_pad), dtype=np.uint8)
+    full[:, :rows] = np.stack(planes)
+    blocks = full.reshape(P, rows_pad // 128, 128, k_pad // 128, 128).transpose(1, 3, 0, 2, 4)
+    return np.ascontiguousarray(blocks)
