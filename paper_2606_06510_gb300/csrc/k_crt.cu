@@ -316,53 +316,45 @@ __device__ __forceinline__ bool crt_fast(const int (&c)[R], int E, const Oz2Modu
 }
 
 // Resident blocks per SM the register budget is sized for: the two-word
-// path fits 64 registers up to r = 10; larger r gets more registers.
-template <int R>
+// path fits 64 registers (four blocks) up to r = 12 in the FAST kernel and
+// up to r = 10 in the element-wise one; the five-limb path (r ≥ 13) takes
+// 128.
+template <int R, bool FAST>
 constexpr int crt_min_blocks() {
-  return R <= 10 ? 4 : (R <= 12 ? 3 : 2);
+  return R <= (FAST ? 12 : 10) ? 4 : (R <= 12 ? 3 : 2);
 }
 
-template <int R>
-__global__ void __launch_bounds__(kCrtThreads, crt_min_blocks<R>())
-    crt_kernel(int64_t m, int64_t n, const __grid_constant__ Oz2Moduli mods, const int16_t* __restrict__ res,
-               int64_t ldr, const int* __restrict__ d, const int* __restrict__ e, double* __restrict__ C,
-               int64_t ldc, int vec_in, int vec_out) {
-  const int64_t row = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) * 2;
-  if (row >= m) return;
-  const bool pair = row + 1 < m;
-  const size_t mstride = static_cast<size_t>(n) * ldr;
-  const int d0 = d[row], d1 = pair ? d[row + 1] : 0;
-  const int16_t* pbase = res + row;
-  double* cbase = C + row;
+// The columns of one thread (two rows, or one at an odd last row): each
+// column's residues are loaded while the previous column is reconstructed,
+// alternating between two buffers.  FAST: both rows present, 4-byte residue
+// loads and 16-byte stores possible; otherwise element-wise accesses.
+// Returns how many outputs were left to Garner's algorithm.
+template <int R, bool FAST>
+__device__ __forceinline__ int crt_columns(int64_t n, int64_t row, bool pair, int d0, int d1,
+                                           const Oz2Moduli& mods, const int16_t* __restrict__ res, int64_t ldr,
+                                           const int* __restrict__ e, double* cbase, int64_t ldc) {
   const int64_t step = gridDim.y;
-  // Two rows' residues of one column, packed (row in the low half).
-  auto load_words = [&](int64_t col, uint32_t (&w)[R]) {
-    const int16_t* p = pbase + col * ldr;
-    if (vec_in && pair) {
+  const int64_t off_step = step * ldr;
+  // Residue matrix k starts at res + k·mstride (the same for every thread,
+  // formed once); this thread's entry of a column is row + col·ldr elements
+  // further.
+  const size_t mstride = static_cast<size_t>(n) * ldr;
+  const int16_t* base[R];
 #pragma unroll
-      for (int k = 0; k < R; ++k) w[k] = __ldg(reinterpret_cast<const uint32_t*>(p + k * mstride));
+  for (int k = 0; k < R; ++k) base[k] = res + k * mstride;
+  // Two rows' residues of one column, packed (row in the low half).
+  auto load_words = [&](int64_t off, uint32_t (&w)[R]) {
+    if (FAST) {
+#pragma unroll
+      for (int k = 0; k < R; ++k) w[k] = __ldg(reinterpret_cast<const uint32_t*>(base[k] + off));
     } else {
 #pragma unroll
       for (int k = 0; k < R; ++k)
-        w[k] = static_cast<uint16_t>(p[k * mstride]) | (pair ? static_cast<uint32_t>(p[k * mstride + 1]) << 16 : 0u);
+        w[k] = static_cast<uint16_t>(base[k][off]) | (pair ? static_cast<uint32_t>(base[k][off + 1]) << 16 : 0u);
     }
   };
-  uint32_t nw[R];
-  int nec = 0;
-  if (static_cast<int64_t>(blockIdx.y) < n) {
-    load_words(blockIdx.y, nw);
-    nec = __ldg(e + blockIdx.y);
-  }
   int pending = 0;
-  for (int64_t col = blockIdx.y; col < n; col += step) {
-    uint32_t w[R];
-#pragma unroll
-    for (int k = 0; k < R; ++k) w[k] = nw[k];
-    const int ec = nec;
-    if (col + step < n) {
-      load_words(col + step, nw);
-      nec = __ldg(e + col + step);
-    }
+  auto column = [&](const uint32_t (&w)[R], int ec, int64_t col) {
     double v[2];
 #pragma unroll
     for (int u = 0; u < 2; ++u) {
@@ -378,58 +370,113 @@ __global__ void __launch_bounds__(kCrtThreads, crt_min_blocks<R>())
       v[u] = val;
     }
     double* out = cbase + col * ldc;
-    if (vec_out && pair) {
+    if (FAST) {
       *reinterpret_cast<double2*>(out) = make_double2(v[0], v[1]);
     } else {
       out[0] = v[0];
       if (pair) out[1] = v[1];
     }
+  };
+  uint32_t wa[R], wb[R];
+  int ea = 0, eb = 0;
+  int64_t col = blockIdx.y, off = col * ldr + row;
+  if (col < n) {
+    load_words(off, wa);
+    ea = __ldg(e + col);
   }
+  while (col < n) {
+    if (col + step < n) {
+      load_words(off + off_step, wb);
+      eb = __ldg(e + col + step);
+    }
+    column(wa, ea, col);
+    col += step;
+    off += off_step;
+    if (col >= n) break;
+    if (col + step < n) {
+      load_words(off + off_step, wa);
+      ea = __ldg(e + col + step);
+    }
+    column(wb, eb, col);
+    col += step;
+    off += off_step;
+  }
+  return pending;
+}
+
+// Rows [row0, row0 + rows) of C.  FAST kernels take row pairs with 4-byte
+// residue loads and 16-byte stores (rows even, residues and C aligned); the
+// other kernel takes any rows element-wise.  The two are separate kernels so
+// that each gets its own register allocation.
+template <int R, bool FAST>
+__global__ void __launch_bounds__(kCrtThreads, crt_min_blocks<R, FAST>())
+    crt_kernel(int64_t row0, int64_t rows, int64_t n, const __grid_constant__ Oz2Moduli mods,
+               const int16_t* __restrict__ res, int64_t ldr, const int* __restrict__ d, const int* __restrict__ e,
+               double* __restrict__ C, int64_t ldc) {
+  const int64_t rel = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) * 2;
+  if (rel >= rows) return;
+  const int64_t row = row0 + rel;
+  const bool pair = rel + 1 < rows;
+  const int d0 = d[row], d1 = pair ? d[row + 1] : 0;
+  double* cbase = C + row;
+  const int pending = crt_columns<R, FAST>(n, row, pair, d0, d1, mods, res, ldr, e, cbase, ldc);
   if (pending == 0) return;
   // Outputs the fast path left to Garner's algorithm (this thread's own).
+  const int64_t step = gridDim.y;
   for (int64_t col = blockIdx.y; col < n; col += step) {
     for (int u = 0; u < (pair ? 2 : 1); ++u) {
       double* q = cbase + col * ldc + u;
       if (__double_as_longlong(*q) != kCrtSentinel) continue;
-      const int16_t* p = pbase + col * ldr + u;
       int c[R];
 #pragma unroll
-      for (int k = 0; k < R; ++k) c[k] = p[k * mstride];
+      for (int k = 0; k < R; ++k) c[k] = res[(k * n + col) * ldr + row + u];
       *q = crt_value<R>(c, -((u ? d1 : d0) + __ldg(e + col)), mods);
     }
   }
 }
 
+// One launch over rows [row0, row0 + rows): x covers row pairs, y strides
+// over the columns, about two waves of resident blocks in all.
+template <int R, bool FAST>
+static cudaError_t launch_crt_rows(cudaStream_t st, int64_t row0, int64_t rows, int64_t n, const Oz2Moduli& mods,
+                                   const int16_t* res, int64_t ldr, const int32_t* d, const int32_t* e, double* C,
+                                   int64_t ldc) {
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int64_t gx = ((rows + 1) / 2 + kCrtThreads - 1) / kCrtThreads;
+  if (gx > 0x7FFFFFFF) return cudaErrorInvalidValue;
+  int64_t gy = (2LL * crt_min_blocks<R, FAST>() * sms + gx - 1) / gx;
+  gy = gy < 1 ? 1 : gy;
+  gy = gy > n ? n : gy;
+  gy = gy > 65535 ? 65535 : gy;
+  count_launch();
+  crt_kernel<R, FAST><<<dim3(static_cast<unsigned>(gx), static_cast<unsigned>(gy)), kCrtThreads, 0, st>>>(
+      row0, rows, n, mods, res, ldr, d, e, C, ldc);
+  return cudaGetLastError();
+}
+
 template <int R>
-static void launch_crt_r(dim3 grid, cudaStream_t st, int64_t m, int64_t n, const Oz2Moduli& mods, const int16_t* res,
-                         int64_t ldr, const int32_t* d, const int32_t* e, double* C, int64_t ldc, int vi, int vo) {
-  crt_kernel<R><<<grid, kCrtThreads, 0, st>>>(m, n, mods, res, ldr, d, e, C, ldc, vi, vo);
+static cudaError_t launch_crt_r(cudaStream_t st, int64_t m, int64_t n, const Oz2Moduli& mods, const int16_t* res,
+                                int64_t ldr, const int32_t* d, const int32_t* e, double* C, int64_t ldc) {
+  const bool vec = (ldr % 2 == 0) && (reinterpret_cast<uintptr_t>(res) % 4 == 0) && (ldc % 2 == 0) &&
+                   (reinterpret_cast<uintptr_t>(C) % 16 == 0);
+  if (!vec) return launch_crt_rows<R, false>(st, 0, m, n, mods, res, ldr, d, e, C, ldc);
+  const int64_t even = m & ~int64_t{1};
+  cudaError_t err = cudaSuccess;
+  if (even > 0) err = launch_crt_rows<R, true>(st, 0, even, n, mods, res, ldr, d, e, C, ldc);
+  if (err == cudaSuccess && even < m) err = launch_crt_rows<R, false>(st, even, 1, n, mods, res, ldr, d, e, C, ldc);
+  return err;
 }
 
 cudaError_t launch_reconstruct(int64_t m, int64_t n, const Oz2Moduli& mods, const int16_t* residues,
                                int64_t ldr, const int32_t* d, const int32_t* e, double* C, int64_t ldc,
                                cudaStream_t st) {
   if (m == 0 || n == 0) return cudaSuccess;
-  int dev = 0, sms = 148;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  // x: row pairs; y: columns strided over gridDim.y, about two waves of
-  // 4 resident blocks per SM in total.
-  const int64_t gx = ((m + 1) / 2 + kCrtThreads - 1) / kCrtThreads;
-  if (gx > 0x7FFFFFFF) return cudaErrorInvalidValue;
-  int64_t gy = (8LL * sms + gx - 1) / gx;
-  gy = gy < 1 ? 1 : gy;
-  gy = gy > n ? n : gy;
-  gy = gy > 65535 ? 65535 : gy;
-  const dim3 grid(static_cast<unsigned>(gx), static_cast<unsigned>(gy));
-  const int vi = (ldr % 2 == 0) && (reinterpret_cast<uintptr_t>(residues) % 4 == 0);
-  const int vo = (ldc % 2 == 0) && (reinterpret_cast<uintptr_t>(C) % 16 == 0);
-  count_launch();
   switch (mods.r) {
 #define OZ2_CRT_CASE(R) \
   case R:               \
-    launch_crt_r<R>(grid, st, m, n, mods, residues, ldr, d, e, C, ldc, vi, vo); \
-    break;
+    return launch_crt_r<R>(st, m, n, mods, residues, ldr, d, e, C, ldc);
     OZ2_CRT_CASE(1) OZ2_CRT_CASE(2) OZ2_CRT_CASE(3) OZ2_CRT_CASE(4) OZ2_CRT_CASE(5) OZ2_CRT_CASE(6)
     OZ2_CRT_CASE(7) OZ2_CRT_CASE(8) OZ2_CRT_CASE(9) OZ2_CRT_CASE(10) OZ2_CRT_CASE(11) OZ2_CRT_CASE(12)
     OZ2_CRT_CASE(13) OZ2_CRT_CASE(14) OZ2_CRT_CASE(15) OZ2_CRT_CASE(16)
@@ -437,7 +484,6 @@ cudaError_t launch_reconstruct(int64_t m, int64_t n, const Oz2Moduli& mods, cons
     default:
       return cudaErrorInvalidValue;
   }
-  return cudaGetLastError();
 }
 
 }  // namespace oz2
