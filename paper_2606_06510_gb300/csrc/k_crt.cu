@@ -270,8 +270,10 @@ __device__ __forceinline__ double finish_words(long long Hs, u64 L, int E) {
 // S = Σ_k c_k W_k (≡ X mod M) and W_k/M = y_k/m_k:
 //  * Y = Σ c_k F_k mod 2^64, read as a signed word, is 2^64·X/M up to
 //    Σ|c_k|/2 units, as long as X/M is not within that of ±1/2;
-//  * q = (S - X)/M is the integer nearest to Σ c_k g_k/2^31 - Y/2^64
-//    (evaluated in units of 2^-11);
+//  * q = (S - X)/M is the integer nearest to Σ c_k g_k/2^18 - Y/2^64
+//    (evaluated in units of 2^-11): with g_k = round(2^18·y_k/m_k) the
+//    first term is within Σ|c_k|·2^-19 < 2^-6 of S/M, and the sum stays a
+//    32-bit integer for |c_k| < m_k;
 //  * L = X mod 2^64 = Σ c_k (W_k mod 2^64) - q·(M mod 2^64), exactly;
 //  * H = ⌊X/2^64⌋ is the integer nearest to Y·round(M/2^51)/2^77 - L/2^64,
 //    from three 32×32 products (the dropped low product is below 1 unit).
@@ -281,18 +283,19 @@ __device__ __forceinline__ double finish_words(long long Hs, u64 L, int E) {
 // returns false and the caller takes Garner's algorithm.
 template <int R>
 __device__ __forceinline__ bool crt_value_w64(const int (&c)[R], int E, const Oz2Moduli& mods, double& out) {
-  long long y0 = 0, l0 = 0, g0 = 0;
+  long long y0 = 0, l0 = 0;
   uint32_t y1 = 0, l1 = 0;
+  int g0 = 0;
 #pragma unroll
   for (int k = 0; k < R; ++k) {
     mad_word(c[k], mods.crt_fl[k], mods.crt_fh[k], y0, y1);
     mad_word(c[k], mods.crt_wl[k], mods.crt_wh[k], l0, l1);
-    g0 += static_cast<long long>(c[k]) * mods.crt_g[k];
+    g0 += c[k] * mods.crt_g[k];
   }
   const uint32_t yl = static_cast<uint32_t>(y0);
   const int yh = static_cast<int>(static_cast<uint32_t>(static_cast<u64>(y0) >> 32) + y1);
   if ((yh ^ (yh >> 31)) >= 0x7FF00000) return false;
-  const int q = (static_cast<int>(g0 >> 20) - (yh >> 21) + 1024) >> 11;
+  const int q = ((g0 >> 7) - (yh >> 21) + 1024) >> 11;
   l0 -= static_cast<long long>(q) * mods.crt_ml;
   l1 -= static_cast<uint32_t>(q) * static_cast<uint32_t>(mods.crt_mlh);
   const u64 L = static_cast<u64>(l0) + (static_cast<u64>(l1) << 32);

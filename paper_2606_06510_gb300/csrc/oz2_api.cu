@@ -186,11 +186,11 @@ static Oz2Moduli build_moduli(int r, int quant) {
     for (int t = 0; t < 5; ++t) c.crtw[k][t] = W[t];
     c.crtf[k] = static_cast<uint32_t>(((static_cast<u64>(y) << 32) + static_cast<u64>(mk / 2)) / static_cast<u64>(mk));
     c.coff[k] = mk * ((32768 + mk - 1) / mk);
-    // Two-word constants: y/m < 1 - 1/m, so both roundings stay below 2^64 and 2^31.
+    // Two-word constants: y/m < 1 - 1/m, so both roundings stay below 2^64 and 2^18.
     const unsigned __int128 fy = ((static_cast<unsigned __int128>(y) << 64) + static_cast<unsigned>(mk / 2)) / mk;
     split_signed_low(static_cast<u64>(fy), &c.crt_fl[k], &c.crt_fh[k]);
     split_signed_low(static_cast<u64>(W[0]) | (static_cast<u64>(W[1]) << 32), &c.crt_wl[k], &c.crt_wh[k]);
-    c.crt_g[k] = static_cast<int>(((static_cast<u64>(y) << 31) + static_cast<u64>(mk / 2)) / static_cast<u64>(mk));
+    c.crt_g[k] = static_cast<int>(((static_cast<u64>(y) << 18) + static_cast<u64>(mk / 2)) / static_cast<u64>(mk));
   }
   u64 M[3] = {1, 0, 0};
   for (int i = 0; i < r; ++i) mul3(M, static_cast<u64>(kModuliAll[i]));

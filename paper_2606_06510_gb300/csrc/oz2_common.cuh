@@ -124,7 +124,7 @@ struct Oz2Moduli {
   // Two-word direct CRT (r ≤ 12, M < 2^112), for signed 32×32→64-bit
   // multiply-adds: F_k = round(2^64·y_k/m_k) mod 2^64 = fh·2^32 + fl and
   // W_k mod 2^64 = wh·2^32 + wl, each with a signed low word;
-  // g_k = round(2^31·y_k/m_k); M mod 2^64 = mlh·2^32 + ml and
+  // g_k = round(2^18·y_k/m_k); M mod 2^64 = mlh·2^32 + ml and
   // round(M/2^51) = m51h·2^32 + m51l (ml, m51l signed).
   int crt_fl[kMaxModuli], crt_fh[kMaxModuli];
   int crt_wl[kMaxModuli], crt_wh[kMaxModuli];

@@ -1,8 +1,10 @@
 """Error budget of the reconstruction's two-word fast path (r ≤ 12).
 
 The CUDA reconstruction finds X from 64-bit fixed-point sums: Y = Σ c_k F_k
-mod 2^64 with F_k = round(2^64·y_k/m_k) approximates 2^64·X/M, and
-H = ⌊X/2^64⌋ is recovered from Y·round(M/2^49)/2^113.  These CPU tests check,
+mod 2^64 with F_k = round(2^64·y_k/m_k) approximates 2^64·X/M, the quotient
+q = (S - X)/M comes from the 32-bit sum Σ c_k g_k with g_k =
+round(2^18·y_k/m_k), and H = ⌊X/2^64⌋ is recovered from
+Y·round(M/2^51)/2^115.  These CPU tests check,
 with exact rational arithmetic on constants built here from their
 definitions, that the worst case over all residues with |c_k| < m_k keeps
 the error of that estimate well below the 1/2 that rounding H tolerates, and
@@ -27,7 +29,7 @@ def constants(r):
         Mk = M // m
         y = pow(Mk % m, -1, m)
         F = ((y << 64) + m // 2) // m
-        g = ((y << 31) + m // 2) // m
+        g = ((y << 18) + m // 2) // m
         out.append((m, y, Mk * y, F, g))
     return M, mods, out
 
@@ -36,20 +38,24 @@ def constants(r):
 def test_fraction_error_budget(r):
     M, mods, cs = constants(r)
     assert M < 2 ** 112
-    mh = (M + (1 << 48)) >> 49
-    assert mh < 2 ** 63
+    mh = (M + (1 << 50)) >> 51
+    assert mh < 2 ** 61
     # |Y - 2^64·X/M| ≤ Σ |c_k|·|F_k - 2^64 y_k/m_k| with |c_k| ≤ m_k - 1.
     err_y = sum((m - 1) * abs(Fraction(F) - Fraction(y << 64, m)) for m, y, _, F, _ in cs)
     assert err_y <= Fraction(1, 2) * sum(m - 1 for m in mods)
     # H estimate in units of 2^64: Y error scaled by M/2^64, plus the rounding
-    # of M/2^49 (|Y| < 2^63), the floor of the high product and of L/2^49.
-    err_h = err_y * Fraction(M, 2 ** 64) / 2 ** 64 + Fraction(2 ** 63, 2 ** 64) * Fraction(1, 2) / 2 ** 15 \
-        + Fraction(2, 2 ** 15)
+    # of M/2^51 (|Y| < 2^63), the dropped low product and the floors of the
+    # high product and of L/2^51 (one unit of 2^51 each).
+    err_h = err_y * Fraction(M, 2 ** 64) / 2 ** 64 + Fraction(2 ** 63, 2 ** 64) * Fraction(1, 2) / 2 ** 13 \
+        + Fraction(3, 2 ** 13)
     assert err_h < Fraction(1, 8), float(err_h)
-    # Quotient estimate Σ c_k g_k/2^31 - Y/2^64: error well below 1/2.
-    err_q = sum((m - 1) * abs(Fraction(g) - Fraction(y << 31, m)) for m, y, _, _, g in cs) / 2 ** 31 \
-        + (err_y + 1) / 2 ** 64 + Fraction(1, 2 ** 31)
-    assert err_q < Fraction(1, 2 ** 12), float(err_q)
+    # Quotient estimate Σ c_k g_k/2^18 - Y/2^64 (q is an integer): error, with
+    # the floors of g0/2^7 and Y/2^53, well below 1/2.
+    err_q = sum((m - 1) * abs(Fraction(g) - Fraction(y << 18, m)) for m, y, _, _, g in cs) / 2 ** 18 \
+        + (err_y + 1) / 2 ** 64 + Fraction(2, 2 ** 11)
+    assert err_q < Fraction(1, 32), float(err_q)
+    # The quotient sum is a 32-bit integer for any |c_k| < m_k.
+    assert sum((m - 1) * g for m, _, _, _, g in cs) < 2 ** 31
     # The margin in Y (2^52) is far above its error.
     assert err_y < 2 ** 40
 
@@ -64,11 +70,12 @@ def word_path(c, r):
     if abs(Ys if Ys >= 0 else ~Ys) >= (1 << 63) - (1 << 52):
         return None
     g0 = sum(ck * g for ck, (_, _, _, _, g) in zip(c, cs))
-    q = (g0 - (Ys >> 33) + (1 << 30)) >> 31
+    assert -2 ** 31 <= g0 < 2 ** 31
+    q = ((g0 >> 7) - (Ys >> 53) + 1024) >> 11
     L = (sum(ck * W for ck, (_, _, W, _, _) in zip(c, cs)) - q * M) & mask
-    mh = (M + (1 << 48)) >> 49
+    mh = (M + (1 << 50)) >> 51
     zh = (Ys * mh) >> 64
-    H = (zh - (L >> 49) + (1 << 14)) >> 15
+    H = (zh - (L >> 51) + 4096) >> 13
     return H * 2 ** 64 + L
 
 
