@@ -6,6 +6,7 @@
 #include <atomic>
 #include <cstdio>
 #include <cstring>
+#include <functional>
 #include <mutex>
 
 #include "oz2_common.cuh"
@@ -17,6 +18,8 @@ namespace oz2 {
 static const int kModuliAll[kMaxModuli] = {1089, 1024, 961, 841, 625, 529, 511, 509,
                                            503,  499,  491, 487, 479, 467, 463, 461};
 constexpr int kTableMax = 20480;  // 2·Σ of all sixteen moduli = 19878 entries
+constexpr int kHostBlocksMax = 8;   // column blocks of one oz2_dgemm_host call
+constexpr int64_t kHostBlockCols = 1024;  // their target width
 
 // Packed E4M3 digit planes of every residue (byte p = plane p), 2m entries
 // per modulus, entry i for the residue (i - kDecBias) mod m; table 0 for A
@@ -222,6 +225,13 @@ struct DeviceState {
   // allocates itself; it keeps freed blocks for reuse (release threshold:
   // unlimited) until oz2_trim_memory.
   cudaMemPool_t pool = nullptr;
+  // oz2_dgemm_host: a stream for copying finished column blocks of C back,
+  // one event per block and one for the last copy, created on first use; the
+  // mutex serialises host-buffer calls on this device, which share them.
+  std::mutex host_mu;
+  cudaStream_t copy_stream = nullptr;
+  cudaEvent_t block_done[kHostBlocksMax] = {};
+  cudaEvent_t copies_done = nullptr;
 };
 static DeviceState g_devs[64];
 static std::mutex g_mu;
@@ -444,9 +454,18 @@ int oz2_workspace_layout(int64_t m, int64_t n, int64_t k, int num_moduli, oz2_ws
   return OZ2_OK;
 }
 
-int oz2_dgemm_ex(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, const double* B, int64_t ldb,
-                 double* C, int64_t ldc, int num_moduli, int quant, int scale, unsigned flags, void* workspace,
-                 size_t ws_bytes, void* stream) {
+// Called after the stages of a column block [c0, c0 + cols) of C are
+// enqueued on the call's stream.
+typedef std::function<cudaError_t(int64_t c0, int64_t cols)> BlockDone;
+
+// Algorithm 1 on the call's stream.  Phase 1 (scan, "+1" pass, scales,
+// deconstruction) covers the whole problem; the residue GEMM, the
+// reconstruction and the fallback then run per column block of `col_block`
+// columns (a multiple of 256; 0 or ≥ n: one block), each followed by
+// `on_block`.  The results do not depend on the blocking.
+static int run_stages(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, const double* B, int64_t ldb,
+                      double* C, int64_t ldc, int num_moduli, int quant, int scale, unsigned flags, void* workspace,
+                      size_t ws_bytes, void* stream, int64_t col_block, const BlockDone* on_block) {
   int st = check_sizes(m, n, k, lda, ldb, ldc);
   if (st) return st;
   if (num_moduli < 1 || num_moduli > kMaxModuli) return OZ2_ERR_UNSUPPORTED_R;
@@ -526,17 +545,33 @@ int oz2_dgemm_ex(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, 
   if (err == cudaSuccess)
     err = launch_deconstruct(m, n, k, mods, ds->table_a, ds->table_b, A, lda, B, ldb, d, e, rf, cf, quant, pa, pb, s);
   mark(5);
-  if (err == cudaSuccess)
-    err = launch_plane_gemm(m, n, L.k_pad, mods, pa, pb, simt ? 2 : 0, res, L.res_ld, nullptr, ds->status, s);
-  mark(6);
-  if (err == cudaSuccess) err = launch_reconstruct(m, n, mods, res, L.res_ld, d, e, C, ldc, s);
-  mark(7);
-  if (err == cudaSuccess) err = launch_fallback_lists(m, n, k, A, lda, B, ldb, rf, cf, misc, C, ldc, s, false);
-  mark(8);
+  // Phase 2 by column blocks (stage timing needs a single block).
+  const int64_t nb = (col_block <= 0 || col_block >= n || ts) ? n : col_block;
+  for (int64_t c0 = 0; c0 < n && err == cudaSuccess; c0 += nb) {
+    const int64_t cols = std::min(nb, n - c0);
+    const uint8_t* pb0 = pb + static_cast<size_t>(c0 / kPlaneRows) * (L.k_pad / kPlaneLine) * L.num_planes *
+                                  static_cast<size_t>(kPlaneBlock);
+    err = launch_plane_gemm(m, cols, L.k_pad, mods, pa, pb0, simt ? 2 : 0, res, L.res_ld, nullptr, ds->status, s);
+    mark(6);
+    if (err == cudaSuccess) err = launch_reconstruct(m, cols, mods, res, L.res_ld, d, e + c0, C + c0 * ldc, ldc, s);
+    mark(7);
+    if (err == cudaSuccess)
+      err = launch_fallback_lists(m, cols, k, A, lda, B + c0 * ldb, ldb, rf, cf + c0, misc, C + c0 * ldc, ldc, s,
+                                  c0 > 0);
+    mark(8);
+    if (err == cudaSuccess && on_block) err = (*on_block)(c0, cols);
+  }
 
   hs.k_slab = static_cast<int>(std::min<int64_t>(kKSlabMerged, L.k_pad));
   if (ts) ts->pending = true;
   return to_status(err);
+}
+
+int oz2_dgemm_ex(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, const double* B, int64_t ldb,
+                 double* C, int64_t ldc, int num_moduli, int quant, int scale, unsigned flags, void* workspace,
+                 size_t ws_bytes, void* stream) {
+  return run_stages(m, n, k, A, lda, B, ldb, C, ldc, num_moduli, quant, scale, flags, workspace, ws_bytes, stream, 0,
+                    nullptr);
 }
 
 int oz2_dgemm(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, const double* B, int64_t ldb,
@@ -567,7 +602,17 @@ int oz2_dgemm_host(int64_t m, int64_t n, int64_t k, const double* hA, int64_t ld
   if (num_moduli < 1 || num_moduli > kMaxModuli) return OZ2_ERR_UNSUPPORTED_R;
   if (m == 0 || n == 0) return OZ2_OK;
   if (!hC || (k > 0 && (!hA || !hB))) return OZ2_ERR_INVALID_ARG;
+  DeviceState* ds = nullptr;
+  if ((st = device_state(&ds)) != OZ2_OK) return st;
+  std::lock_guard<std::mutex> host_lock(ds->host_mu);
+  if (!ds->copy_stream) {
+    if (cudaStreamCreateWithFlags(&ds->copy_stream, cudaStreamNonBlocking) != cudaSuccess) return OZ2_ERR_CUDA;
+    for (int i = 0; i < kHostBlocksMax; ++i)
+      if (cudaEventCreateWithFlags(&ds->block_done[i], cudaEventDisableTiming) != cudaSuccess) return OZ2_ERR_CUDA;
+    if (cudaEventCreateWithFlags(&ds->copies_done, cudaEventDisableTiming) != cudaSuccess) return OZ2_ERR_CUDA;
+  }
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaStream_t cs = ds->copy_stream;
   const size_t bA = align256(sizeof(double) * m * k), bB = align256(sizeof(double) * k * n),
                bC = align256(sizeof(double) * m * n);
   const size_t ws = k > 0 ? oz2_workspace_size(m, n, k, num_moduli) : 0;
@@ -584,11 +629,30 @@ int oz2_dgemm_host(int64_t m, int64_t n, int64_t k, const double* hA, int64_t ld
     err = copy_matrix(dA, m, hA, lda, m, k, cudaMemcpyHostToDevice, s);
     if (err == cudaSuccess) err = copy_matrix(dB, k, hB, ldb, k, n, cudaMemcpyHostToDevice, s);
   }
-  if (err == cudaSuccess)
-    st = oz2_dgemm_ex(m, n, k, dA, m, dB, std::max<int64_t>(1, k), dC, m, num_moduli, OZ2_QUANT_TZ, OZ2_SCALE_R2,
-                      0, k > 0 ? buf + bA + bB + bC : nullptr, ws, stream);
-  if (err == cudaSuccess && st == OZ2_OK)
-    err = copy_matrix(hC, ldc, dC, m, m, n, cudaMemcpyDeviceToHost, s);
+  // C goes back by column blocks on the copy stream, each as soon as its
+  // reconstruction and fallback are done, so that the copies overlap the
+  // residue GEMM of the blocks after it.
+  const int64_t nblk = std::max<int64_t>(1, std::min<int64_t>(kHostBlocksMax, (n + kHostBlockCols / 2) / kHostBlockCols));
+  const int64_t col_block = ((n + nblk - 1) / nblk + 255) / 256 * 256;
+  int blk = 0;
+  const BlockDone copy_back = [&](int64_t c0, int64_t cols) -> cudaError_t {
+    cudaError_t e = cudaEventRecord(ds->block_done[blk], s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(cs, ds->block_done[blk], 0);
+    if (e == cudaSuccess) e = copy_matrix(hC + c0 * ldc, ldc, dC + c0 * m, m, m, cols, cudaMemcpyDeviceToHost, cs);
+    ++blk;
+    return e;
+  };
+  if (err == cudaSuccess) {
+    if (k > 0) {
+      st = run_stages(m, n, k, dA, m, dB, k, dC, m, num_moduli, OZ2_QUANT_TZ, OZ2_SCALE_R2, 0,
+                      buf + bA + bB + bC, ws, stream, col_block, &copy_back);
+    } else {  // C = 0
+      err = cudaMemsetAsync(dC, 0, sizeof(double) * m * n, s);
+      if (err == cudaSuccess) err = copy_back(0, n);
+    }
+  }
+  // The buffers are released once the copies have read them.
+  if (cudaEventRecord(ds->copies_done, cs) == cudaSuccess) cudaStreamWaitEvent(s, ds->copies_done, 0);
   cudaFreeAsync(buf, s);
   if (cudaStreamSynchronize(s) != cudaSuccess && err == cudaSuccess) err = cudaErrorUnknown;
   if (st != OZ2_OK) return st;

@@ -1,0 +1,75 @@
+"""The host-buffer entry oz2_dgemm_host against the CPU oracle, bit for bit.
+
+For wide C the entry runs the residue GEMM, the reconstruction and the
+fallback by column blocks of about 1024 columns and copies each block of C
+back while the next one is computed; the result must not depend on that.
+"""
+import numpy as np
+import pytest
+
+import workloads as wl
+from helpers import ensure_built
+from oracle import ozaki2 as orc
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def oz():
+    ensure_built()
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2606_06510_gb300 as oz
+    oz.lib()
+    return oz
+
+
+def pinned_colmajor(x):
+    """A pinned CPU tensor holding x column-major (stride 1 down a column)."""
+    import torch
+    t = torch.empty((x.shape[1], x.shape[0]), dtype=torch.float64, pin_memory=True)
+    t.copy_(torch.from_numpy(np.ascontiguousarray(x.T)))
+    return t.t()
+
+
+def assert_same(got, want):
+    same = (got == want) | (np.isnan(got) & np.isnan(want))
+    assert same.all(), f"{(~same).sum()} entries differ; first {np.argwhere(~same)[0]}"
+    assert np.array_equal(np.signbit(got), np.signbit(want))
+
+
+def test_column_blocks_with_fallback_and_padded_c(oz):
+    """n = 2600: blocks of 1024, 1024 and 552 columns.  A fallback row (2^300)
+    and a zero row in A; a NaN column in the second block and a 2^-200 column
+    in the last one; C with leading dimension m + 5."""
+    import torch
+    m, n, k = 300, 2600, 70
+    A = np.array(wl.random_matrix(m, k, 1.0, 7100), order="F")
+    B = np.array(wl.random_matrix(k, n, 1.0, 7200), order="F")
+    A[7, :] *= 2.0 ** 300
+    A[123, :] = 0.0
+    B[3, 1500] = np.nan
+    B[:, 2599] *= 2.0 ** -200
+    want = orc.oz2_dgemm(A, B, 12).C
+    C = torch.full((n, m + 5), 7.0, dtype=torch.float64, pin_memory=True).t()[:m]
+    oz.oz2_dgemm_host(pinned_colmajor(A), pinned_colmajor(B), C)
+    assert_same(C.numpy(), want)
+    assert oz.oz2_check_device_status() == 0
+
+
+def test_one_block_from_numpy(oz):
+    m, n, k = 257, 300, 129
+    A = np.array(wl.random_matrix(m, k, 0.5, 7300), order="F")
+    B = np.array(wl.random_matrix(k, n, 0.5, 7400), order="F")
+    C = oz.oz2_dgemm_host(A, B, num_moduli=9)
+    assert_same(C, orc.oz2_dgemm(A, B, 9).C)
+
+
+def test_empty_k_gives_zero(oz):
+    m, n = 40, 1800
+    A = np.zeros((m, 0), order="F")
+    B = np.zeros((0, n), order="F")
+    C = np.full((m, n), 3.0, order="F")
+    oz.oz2_dgemm_host(A, B, C)
+    assert np.array_equal(C, np.zeros((m, n))) and not np.signbit(C).any()
