@@ -141,18 +141,7 @@ static Oz2Moduli build_moduli(int r, int quant) {
     c.sq_base[i] = isqrt_exact(m);
     c.plane_off[i] = plane;
     plane += c.sq_base[i] ? 2 : 3;
-    c.table_off[i] = toff;
     toff += m;
-    int sh = 31 - __builtin_clz(static_cast<unsigned>(m - 1));
-    u64 num = 1ull << (32 + sh);
-    c.magic[i] = static_cast<uint32_t>((num + m - 1) / m);
-    c.magic_sh[i] = sh;
-    for (int j = 0; j < 4; ++j) {
-      u64 v = 1;
-      for (int t = 0; t < j; ++t) v = (v << 16) % m;
-      c.limb[i][j] = static_cast<int>(v);
-    }
-    c.negoff[i] = m * static_cast<int>(((1u << 28) + m - 1) / m);
     c.goff[i] = m * static_cast<int>(((1u << 27) + m - 1) / m);
     long long P = 1;  // product of the earlier moduli, mod m
     for (int t = 0; t < i; ++t) {

@@ -101,11 +101,6 @@ struct Oz2Moduli {
   int m[kMaxModuli];
   int sq_base[kMaxModuli];      // s for m = s², 0 for nonsquare
   int plane_off[kMaxModuli];    // first plane of modulus i
-  int table_off[kMaxModuli];    // first entry of modulus i in the plane table
-  uint32_t magic[kMaxModuli];   // ⌈2^(32+sh)/m⌉, sh = ⌊log2(m-1)⌋
-  int magic_sh[kMaxModuli];
-  int limb[kMaxModuli][4];      // 2^(16j) mod m
-  int negoff[kMaxModuli];       // multiple of m ≥ 2^28 (sign handling)
   // Garner (Eq. garner): pmod[k][j] = (m_0 ⋯ m_{j-1}) mod m_k for j < k,
   // inv[k] = (m_0 ⋯ m_{k-1})^-1 mod m_k, goff[k] = multiple of m_k ≥ 2^27.
   int pmod[kMaxModuli][kMaxModuli];
