@@ -73,3 +73,33 @@ def test_empty_k_gives_zero(oz):
     C = np.full((m, n), 3.0, order="F")
     oz.oz2_dgemm_host(A, B, C)
     assert np.array_equal(C, np.zeros((m, n))) and not np.signbit(C).any()
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_randomised_wide_problems(oz, seed):
+    """Seeded wide problems (n from 1400 to 3400, so two to three column
+    blocks with a ragged last one), r from 1 to 16, φ from 0 to 5, and
+    planted special rows of A and columns of B in random blocks."""
+    rng = np.random.default_rng(8000 + seed)
+    m = int(rng.integers(1, 200))
+    n = int(rng.integers(1400, 3400))
+    k = int(rng.integers(1, 120))
+    r = int(rng.integers(1, 17))
+    phi = float(rng.uniform(0.0, 5.0))
+    A = np.array(wl.random_matrix(m, k, phi, 8100 + seed), order="F")
+    B = np.array(wl.random_matrix(k, n, phi, 8200 + seed), order="F")
+    for _ in range(int(rng.integers(0, 3))):
+        i = int(rng.integers(0, m))
+        A[i, :] *= 2.0 ** (300 if rng.integers(0, 2) else -300)
+    for _ in range(int(rng.integers(0, 4))):
+        j, kind = int(rng.integers(0, n)), int(rng.integers(0, 3))
+        if kind == 0:
+            B[:, j] = 0.0
+        elif kind == 1:
+            B[int(rng.integers(0, k)), j] = np.inf
+        else:
+            B[:, j] *= 2.0 ** -250
+    want = orc.oz2_dgemm(A, B, r).C
+    got = oz.oz2_dgemm_host(A, B, num_moduli=r)
+    assert_same(got, want)
+    assert oz.oz2_check_device_status() == 0
