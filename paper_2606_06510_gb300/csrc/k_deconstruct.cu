@@ -165,11 +165,61 @@ __device__ __forceinline__ void load8(const OperandView& X, int64_t row, int64_t
 // more, since the second term is below y/2^30 < 1; so Y - 4qm = 4(y - qm) is
 // the byte offset of the entry for y mod m in a table whose 2m entries
 // start m entries before it.  The table is rotated by kDecBias.
+// E4M3 codes of two integer-valued floats, `lo` in bits 0-7 and `hi` in
+// bits 8-15 (exact: both are integers of magnitude at most 16).
+__device__ __forceinline__ uint32_t e4m3x2(float lo, float hi) {
+  uint16_t r;
+  asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+// The integer v (|v| < 2^22) as a float: 1.5·2^23 + v has ulp 1.
+__device__ __forceinline__ float small_int_float(uint32_t biased) {
+  return __int_as_float(static_cast<int>(biased)) - 12582912.0f;
+}
+
+// Square modulus m = s² (§2.5, balanced base s): the digits of the centred
+// residue c are computed, not looked up.  With u = c + h0 + s·h1 ≥ 0,
+// d0 = (u mod s) - h0 and d1 = ⌊u/s⌋ - h1.  u = ((y + E) mod m) + h0 + s·h1 -
+// ⌊m/2⌋, since c = ((x + ⌊m/2⌋) mod m) - ⌊m/2⌋ for x = Ã mod m = (y - B)
+// mod m.  (y + E) mod m comes from the same shifted magic quotient as the
+// table index, corrected once.
+template <int I>
+__device__ __forceinline__ void square_digits(const uint32_t (&b)[kElems], const uint32_t (&u1)[kElems],
+                                              const uint32_t (&u2)[kElems], const int (&u3)[kElems],
+                                              uint8_t* dst) {
+  constexpr ModConst mc = mod_const(I);
+  constexpr int kShift = mc.sq_h0 + mc.s * mc.sq_h1 - mc.m / 2;  // u - (y + E) mod m, ≥ 0
+  float f0[kElems], f1[kElems];
+#pragma unroll
+  for (int e = 0; e < kElems; ++e) {
+    const uint32_t Y = b[e] + 4 * mc.sq_e + u1[e] * mc.limb1 + u2[e] * mc.limb2 +
+                       static_cast<uint32_t>(u3[e]) * mc.limb3;
+    const uint32_t q = __umulhi(Y, mc.magic);
+    int off = static_cast<int>(Y - q * static_cast<uint32_t>(4 * mc.m));  // 4·((y + E) mod m) or that - 4m
+    off += off < 0 ? 4 * mc.m : 0;
+    const uint32_t u = (static_cast<uint32_t>(off) >> 2) + kShift;
+    const uint32_t a1 = mc.s == 32 ? u >> 5 : __umulhi(u, mc.sq_magic);
+    const uint32_t a0 = u - a1 * static_cast<uint32_t>(mc.s);
+    f0[e] = small_int_float(a0 + (0x4B400000u - mc.sq_h0));
+    f1[e] = small_int_float(a1 + (0x4B400000u - mc.sq_h1));
+  }
+  uint8_t* pdst = dst + mc.plane_off * kPlaneBlock;
+  *reinterpret_cast<uint2*>(pdst) = make_uint2(__byte_perm(e4m3x2(f0[0], f0[1]), e4m3x2(f0[2], f0[3]), 0x5410),
+                                               __byte_perm(e4m3x2(f0[4], f0[5]), e4m3x2(f0[6], f0[7]), 0x5410));
+  *reinterpret_cast<uint2*>(pdst + kPlaneBlock) =
+      make_uint2(__byte_perm(e4m3x2(f1[0], f1[1]), e4m3x2(f1[2], f1[3]), 0x5410),
+                 __byte_perm(e4m3x2(f1[4], f1[5]), e4m3x2(f1[6], f1[7]), 0x5410));
+}
+
 template <int I>
 __device__ __forceinline__ void planes_one(const uint32_t (&b)[kElems], const uint32_t (&u1)[kElems],
                                            const uint32_t (&u2)[kElems], const int (&u3)[kElems],
                                            const uint32_t* table, uint8_t* dst) {
   constexpr ModConst mc = mod_const(I);
+  if constexpr (mc.s != 0) {
+    square_digits<I>(b, u1, u2, u3, dst);
+    return;
+  }
   const char* centre = reinterpret_cast<const char*>(table + mc.table_off + mc.m);
   uint32_t w[kElems];
 #pragma unroll

@@ -17,13 +17,14 @@ namespace oz2 {
 // extension primes used for r = 13..16 (nonsquare, < 513).
 static const int kModuliAll[kMaxModuli] = {1089, 1024, 961, 841, 625, 529, 511, 509,
                                            503,  499,  491, 487, 479, 467, 463, 461};
-constexpr int kTableMax = 20480;  // 2·Σ of all sixteen moduli = 19878 entries
+constexpr int kTableMax = 20480;  // 2·Σ of the ten nonsquare moduli = 9740 entries
 constexpr int kHostBlocksMax = 8;   // column blocks of one oz2_dgemm_host call
 constexpr int64_t kHostBlockCols = 1024;  // their target width
 
-// Packed E4M3 digit planes of every residue (byte p = plane p), 2m entries
-// per modulus, entry i for the residue (i - kDecBias) mod m; table 0 for A
-// (last nonsquare plane pre-scaled by -16), table 1 for B.
+// Packed E4M3 digit planes of every residue (byte p = plane p) of the
+// nonsquare moduli, 2m entries per modulus, entry i for the residue
+// (i - kDecBias) mod m; table 0 for A (last plane pre-scaled by -16), table 1
+// for B.
 static __device__ uint32_t g_plane_table[2][kTableMax];
 // Device status block (sticky status word, fallback counts, scale summary).
 static __device__ Oz2Device g_status;
@@ -141,7 +142,7 @@ static Oz2Moduli build_moduli(int r, int quant) {
     c.sq_base[i] = isqrt_exact(m);
     c.plane_off[i] = plane;
     plane += c.sq_base[i] ? 2 : 3;
-    toff += m;
+    if (!c.sq_base[i]) toff += m;  // the digit-plane table holds nonsquare moduli only
     c.goff[i] = m * static_cast<int>(((1u << 27) + m - 1) / m);
     long long P = 1;  // product of the earlier moduli, mod m
     for (int t = 0; t < i; ++t) {
@@ -268,6 +269,7 @@ static int device_state(DeviceState** out) {
       int off = 0;
       for (int i = 0; i < kMaxModuli; ++i) {
         const int m = kModuliAll[i];
+        if (isqrt_exact(m)) continue;  // square moduli compute their digits
         for (int j = 0; j < 2 * m; ++j) {
           const int r = floor_mod(j - kDecBias % m, m);
           const int d = r > m - 1 - m / 2 ? r - m : r;  // centred residue

@@ -31,19 +31,25 @@ constexpr int kKSlabMerged = 4096;
 constexpr int kModuliList[kMaxModuli] = {1089, 1024, 961, 841, 625, 529, 511, 509,
                                          503,  499,  491, 487, 479, 467, 463, 461};
 
-// The deconstruction's digit-plane table holds 2m entries per modulus
-// (entry i: the planes of the residue (i - kDecBias) mod m), so that a
-// quotient one too large, and the bias that keeps the residue sum positive,
-// cost nothing at the lookup.
+// The deconstruction's digit-plane table holds 2m entries per nonsquare
+// modulus (entry i: the planes of the residue (i - kDecBias) mod m), so that
+// a quotient one too large, and the bias that keeps the residue sum
+// positive, cost nothing at the lookup.  Square moduli compute their digits.
 constexpr int kDecBias = 1 << 25;
 
 struct ModConst {
   int m;
   int s;          // square base, 0 for nonsquare moduli
   int plane_off;  // first plane of this modulus
-  int table_off;  // first of this modulus's 2m entries in the digit-plane table
+  int table_off;  // nonsquare: first of its 2m entries in the digit-plane table
   uint32_t limb1, limb2, limb3;  // 4·(2^16 mod m), 4·(2^32 mod m), 4·(2^48 mod m)
   uint32_t magic;                // ⌈2^30/m⌉
+  // Square moduli (digits computed, not looked up): E = (⌊m/2⌋ - kDecBias)
+  // mod m, the digit offsets h0 = ⌊s/2⌋ and h1 = ⌈(⌊m/2⌋ - h0)/s⌉, and
+  // ⌈2^32/s⌉.
+  uint32_t sq_e;
+  int sq_h0, sq_h1;
+  uint32_t sq_magic;
 };
 
 constexpr int ce_isqrt(int m) {
@@ -76,7 +82,7 @@ constexpr ModConst mod_const(int i) {
   int plane = 0, toff = 0;
   for (int j = 0; j < i; ++j) {
     plane += ce_isqrt(kModuliList[j]) ? 2 : 3;
-    toff += kModuliList[j];
+    toff += ce_isqrt(kModuliList[j]) ? 0 : kModuliList[j];  // the table holds nonsquare moduli only
   }
   const int m = kModuliList[i];
   c.m = m;
@@ -88,6 +94,13 @@ constexpr ModConst mod_const(int i) {
   c.limb2 = static_cast<uint32_t>(4 * ((1ull << 32) % um));
   c.limb3 = static_cast<uint32_t>(4 * ((1ull << 48) % um));
   c.magic = static_cast<uint32_t>(((1ull << 30) + um - 1) / um);
+  if (c.s) {
+    const int H = m / 2;
+    c.sq_e = static_cast<uint32_t>(((H - kDecBias) % m + m) % m);
+    c.sq_h0 = c.s / 2;
+    c.sq_h1 = (H - c.sq_h0 + c.s - 1) / c.s;
+    c.sq_magic = static_cast<uint32_t>(((1ull << 32) + c.s - 1) / static_cast<unsigned long long>(c.s));
+  }
   return c;
 }
 
@@ -126,7 +139,7 @@ struct Oz2Moduli {
   int crt_g[kMaxModuli];
   int crt_ml, crt_mlh;
   int crt_m51l, crt_m51h;
-  int table_entries;            // 2·Σ m_i (digit-plane table, 2m entries per modulus)
+  int table_entries;            // 2·Σ m_i over the nonsquare moduli (digit-plane table)
 };
 
 // Per-device status block (in device global memory, owned by oz2_api.cu).
