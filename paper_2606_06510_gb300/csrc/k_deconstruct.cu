@@ -79,6 +79,39 @@ __device__ __forceinline__ unsigned long long quantise_abs(const Split& s, int d
   return q;
 }
 
+// Truncating quantisation (Eq. scale, TZ) of one entry into the limbs the
+// residue sums take: Ã = trunc(x·2^d) as a 64-bit two's complement word,
+// for rows with d ≤ kTzFastMaxD, split into
+// b = 4·(bits 0-15 + kDecBias), bits 16-31, bits 32-47 and the signed bits
+// 48-63.  With x = ±M·2^(sh - d), M < 2^53, Ã = ±⌊M·2^10 / 2^(10 - sh)⌋: the
+// significand is shifted up by 10 (below 2^63) and then right by r = 10 - sh
+// with clamping funnel shifts, so zeros, subnormals and entries that shift
+// out entirely need no branch.  That needs sh ≤ 9: a normal x has M ≥ 2^52
+// and |Ã| < 2^62, and a subnormal one has sh = d - 1074 ≤ 9 for
+// d ≤ kTzFastMaxD (rows with a larger scale, whose largest entry is itself
+// subnormal, take the general path).  d = -4096 gives Ã = 0 for any x.
+constexpr int kTzFastMaxD = 1083;
+__device__ __forceinline__ void quantise_tz_limbs(double x, int d, uint32_t& b, uint32_t& u1, uint32_t& u2,
+                                                  int& u3) {
+  const uint32_t hi = static_cast<uint32_t>(__double2hiint(x)), lo = static_cast<uint32_t>(__double2loint(x));
+  const int E = static_cast<int>((hi >> 20) & 0x7FFu);
+  const uint32_t mh = (hi & 0xFFFFFu) | (E ? 0x100000u : 0u);  // M = mh·2^32 + lo
+  const uint32_t r = static_cast<uint32_t>(10 + 1075 - max(E, 1) - d);
+  const uint32_t ph = __funnelshift_l(lo, mh, 10), pl = lo << 10;  // M·2^10
+  const bool wide = r >= 32;
+  const uint32_t x1 = wide ? 0u : ph, x0 = wide ? ph : pl, rr = wide ? r - 32 : r;
+  const uint32_t al = __funnelshift_rc(x0, x1, rr), ah = __funnelshift_rc(x1, 0u, rr);
+  const uint32_t sgn = static_cast<uint32_t>(static_cast<int>(hi) >> 31);  // 0 or all ones
+  const unsigned long long t = ((static_cast<unsigned long long>(ah ^ sgn) << 32) | (al ^ sgn)) -
+                               static_cast<unsigned long long>(static_cast<long long>(static_cast<int>(sgn)));
+  const uint32_t tl = static_cast<uint32_t>(t);
+  const int th = static_cast<int>(t >> 32);
+  b = ((tl << 2) & 0x3FFFCu) | (4u * kDecBias);
+  u1 = tl >> 16;
+  u2 = static_cast<uint32_t>(th) & 0xFFFFu;
+  u3 = th >> 16;
+}
+
 // ⌈log2 |v|⌉ for finite nonzero v.
 __device__ __forceinline__ int ceil_log2_abs(const Split& s) {
   int bl = 64 - __clzll(static_cast<long long>(s.M));
@@ -288,7 +321,8 @@ __global__ void __launch_bounds__(TileShape<MODE>::kThreads, TileShape<MODE>::kB
                   : X.out + ((static_cast<size_t>(row / kPlaneRows) * (k_pad / kPlaneLine) + l0 / kPlaneLine) *
                                  num_planes(R) * kPlaneBlock +
                              (row % kPlaneRows) * kPlaneLine + l0 % kPlaneLine);
-    if (zero_row) {
+    const bool fast_tz = MODE == 1 && !rn && ex <= kTzFastMaxD;
+    if (zero_row && !fast_tz) {  // the fast truncating path zeroes through its scale
 #pragma unroll
       for (int e = 0; e < kElems; ++e) x[e] = 0.0;
     }
@@ -304,17 +338,23 @@ __global__ void __launch_bounds__(TileShape<MODE>::kThreads, TileShape<MODE>::kB
       // into three unsigned 16-bit limbs and a signed top limb.
       uint32_t b[kElems], u1[kElems], u2[kElems];
       int u3[kElems];
+      if (fast_tz) {
+        const int d = zero_row ? -4096 : ex;
 #pragma unroll
-      for (int e = 0; e < kElems; ++e) {
-        const Split sp = split_double(x[e]);
-        const unsigned long long a = quantise_abs(sp, ex, rn != 0);
-        const unsigned long long t = sp.neg ? 0ull - a : a;
-        const uint32_t lo = static_cast<uint32_t>(t);
-        const int hi = static_cast<int>(t >> 32);
-        b[e] = ((lo << 2) & 0x3FFFCu) | (4u * kDecBias);
-        u1[e] = lo >> 16;
-        u2[e] = static_cast<uint32_t>(hi) & 0xFFFFu;
-        u3[e] = hi >> 16;
+        for (int e = 0; e < kElems; ++e) quantise_tz_limbs(x[e], d, b[e], u1[e], u2[e], u3[e]);
+      } else {
+#pragma unroll
+        for (int e = 0; e < kElems; ++e) {
+          const Split sp = split_double(x[e]);
+          const unsigned long long a = quantise_abs(sp, ex, rn != 0);
+          const unsigned long long t = sp.neg ? 0ull - a : a;
+          const uint32_t lo = static_cast<uint32_t>(t);
+          const int hi = static_cast<int>(t >> 32);
+          b[e] = ((lo << 2) & 0x3FFFCu) | (4u * kDecBias);
+          u1[e] = lo >> 16;
+          u2[e] = static_cast<uint32_t>(hi) & 0xFFFFu;
+          u3[e] = hi >> 16;
+        }
       }
       planes_all(std::make_integer_sequence<int, R>{}, b, u1, u2, u3, table, dst);
     }

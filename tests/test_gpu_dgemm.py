@@ -133,6 +133,25 @@ def test_integer_inputs_exact(oz):
     assert np.array_equal(C, A @ B)
 
 
+@pytest.mark.parametrize("quant", ["tz", "rn"])
+def test_subnormal_rows(oz, quant):
+    """Rows of A whose entries are all subnormal: no row is out of range of
+    the others, so none falls back, and their scales exceed 1083 (the
+    deconstruction's general quantisation path).  A normal row and a zero
+    row sit beside them."""
+    m, n, k = 70, 90, 130
+    A = np.array(wl.random_matrix(m, k, 0.5, 9100), order="F") * 2.0 ** -1060
+    A[5, :] = np.array(wl.random_matrix(1, k, 0.5, 9101))[0] * 2.0 ** -1000   # normal, 60 binades up
+    A[9, :] = 0.0
+    assert np.abs(A[10]).max() < 2.2250738585072014e-308 and np.abs(A[10]).max() > 0
+    B = np.array(wl.random_matrix(k, n, 0.5, 9200), order="F")
+    res = orc.oz2_dgemm(A, B, 12, quant=quant)
+    C, v = run_ex(oz, A, B, 12, quant=quant)
+    assert v["d"].max() > 1083
+    assert np.array_equal(v["d"], res.d) and np.array_equal(v["e"], res.e)
+    assert_same(C, res.C)
+
+
 def test_bench_workload_full_size_sampled(oz):
     """4096³, r = 12, φ = 0.5: the configuration bench.py times."""
     w = wl.WORKLOADS["dgemm_4096"]
