@@ -43,7 +43,7 @@ GEMM_SOURCE = os.path.join(ROOT, "paper_2606_06510_gb300", "csrc", "k_gemm.cu")
 # DRAM read+write bytes of one residue-GEMM launch, from the ncu capture in
 # profiles/residue_gemm_dgemm_4096.md; reported only while the kernel source
 # is the one the counters were taken on.
-GEMM_TRAFFIC = {"workload": "dgemm_4096", "num_moduli": 12, "bytes": 2.0916e9,
+GEMM_TRAFFIC = {"workload": "dgemm_4096", "num_moduli": 12, "bytes": 2.0393e9,
                 "sha256": "74d5fa0c2ee816a4e02fac3c1ff584b323bc2d7665487cbcf24bbd150441ec14"}
 
 
