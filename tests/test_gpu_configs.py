@@ -93,3 +93,16 @@ def test_gemv_batch16_character(oz):
     got = run(oz, A, B, w.r)
     check(got, res)
     assert cref.scaled_error(got["C"], A, B, rows=np.arange(0, 1500, 97)) <= 1e-15
+
+
+def test_very_long_k_many_slabs(oz):
+    """k = 262144: eight K-slabs for the square moduli and 64 for the merged
+    nonsquare ones, so the partial residue is carried in the accumulators
+    many times over; the "+1" pass clamp is at its small end (c = 3)."""
+    m, n, k = 9, 7, 262144  # one ragged tile: the slab logic is per tile
+    A = np.array(wl.random_matrix(m, k, 0.5, 9300), order="F")
+    B = np.array(wl.random_matrix(k, n, 0.5, 9400), order="F")
+    res = orc.oz2_dgemm(A, B, 12)
+    got = run(oz, A, B, 12)
+    check(got, res)
+    assert cref.scaled_error(got["C"], A, B, rows=np.arange(m)) <= 1e-15
