@@ -108,11 +108,11 @@ int oz2_dgemm(int64_t m, int64_t n, int64_t k,
  * workspace are allocated and freed stream-ordered inside the call, from the
  * library's memory pool.  A contiguous matrix (ld = rows) moves in one
  * linear copy, any other in a pitched copy.  For wide C (n ≥ 1536) the
- * residue GEMM, reconstruction and fallback run by column blocks of about
- * 1024 columns, and each block of C is copied back on a library-owned copy
- * stream while the next block is computed; the result is the same as
- * unblocked.  Host-buffer calls on one device share that stream and are
- * serialised. */
+ * residue GEMM, reconstruction and fallback run by column blocks (a last
+ * block of 256 columns, the others 768 to 1536 wide), and each block of C
+ * is copied back on a library-owned copy stream while the next block is
+ * computed; the result is the same as unblocked.  Host-buffer calls on one
+ * device share that stream and are serialised. */
 int oz2_dgemm_host(int64_t m, int64_t n, int64_t k,
                    const double* h_A, int64_t lda,
                    const double* h_B, int64_t ldb,

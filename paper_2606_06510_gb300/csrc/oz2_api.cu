@@ -3,6 +3,7 @@
 // Algorithm 1 (scan → "+1" pass and scales → deconstruct → residue GEMMs →
 // Garner/unscale → native fallback).
 #include <algorithm>
+#include <cmath>
 #include <atomic>
 #include <cstdio>
 #include <cstring>
@@ -19,7 +20,6 @@ static const int kModuliAll[kMaxModuli] = {1089, 1024, 961, 841, 625, 529, 511, 
                                            503,  499,  491, 487, 479, 467, 463, 461};
 constexpr int kTableMax = 20480;  // 2·Σ of the ten nonsquare moduli = 9740 entries
 constexpr int kHostBlocksMax = 8;   // column blocks of one oz2_dgemm_host call
-constexpr int64_t kHostBlockCols = 1024;  // their target width
 
 // Packed E4M3 digit planes of every residue (byte p = plane p) of the
 // nonsquare moduli, 2m entries per modulus, entry i for the residue
@@ -449,14 +449,20 @@ int oz2_workspace_layout(int64_t m, int64_t n, int64_t k, int num_moduli, oz2_ws
 // enqueued on the call's stream.
 typedef std::function<cudaError_t(int64_t c0, int64_t cols)> BlockDone;
 
+// Column blocks of C: widths[0..count), each a multiple of 256 but the last.
+struct ColumnBlocks {
+  int count = 0;
+  int64_t widths[kHostBlocksMax] = {};
+};
+
 // Algorithm 1 on the call's stream.  Phase 1 (scan, "+1" pass, scales,
 // deconstruction) covers the whole problem; the residue GEMM, the
-// reconstruction and the fallback then run per column block of `col_block`
-// columns (a multiple of 256; 0 or ≥ n: one block), each followed by
-// `on_block`.  The results do not depend on the blocking.
+// reconstruction and the fallback then run per column block (all of C when
+// `blocks` is null), each followed by `on_block`.  The results do not depend
+// on the blocking.
 static int run_stages(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, const double* B, int64_t ldb,
                       double* C, int64_t ldc, int num_moduli, int quant, int scale, unsigned flags, void* workspace,
-                      size_t ws_bytes, void* stream, int64_t col_block, const BlockDone* on_block) {
+                      size_t ws_bytes, void* stream, const ColumnBlocks* blocks, const BlockDone* on_block) {
   int st = check_sizes(m, n, k, lda, ldb, ldc);
   if (st) return st;
   if (num_moduli < 1 || num_moduli > kMaxModuli) return OZ2_ERR_UNSUPPORTED_R;
@@ -537,9 +543,11 @@ static int run_stages(int64_t m, int64_t n, int64_t k, const double* A, int64_t 
     err = launch_deconstruct(m, n, k, mods, ds->table_a, ds->table_b, A, lda, B, ldb, d, e, rf, cf, quant, pa, pb, s);
   mark(5);
   // Phase 2 by column blocks (stage timing needs a single block).
-  const int64_t nb = (col_block <= 0 || col_block >= n || ts) ? n : col_block;
-  for (int64_t c0 = 0; c0 < n && err == cudaSuccess; c0 += nb) {
-    const int64_t cols = std::min(nb, n - c0);
+  const bool blocked = blocks && blocks->count > 1 && !ts;
+  const int nblk = blocked ? blocks->count : 1;
+  int64_t c0 = 0;
+  for (int bi = 0; bi < nblk && err == cudaSuccess; ++bi) {
+    const int64_t cols = blocked ? blocks->widths[bi] : n;
     const uint8_t* pb0 = pb + static_cast<size_t>(c0 / kPlaneRows) * (L.k_pad / kPlaneLine) * L.num_planes *
                                   static_cast<size_t>(kPlaneBlock);
     err = launch_plane_gemm(m, cols, L.k_pad, mods, pa, pb0, simt ? 2 : 0, res, L.res_ld, nullptr, ds->status, s);
@@ -551,6 +559,7 @@ static int run_stages(int64_t m, int64_t n, int64_t k, const double* A, int64_t 
                                   c0 > 0);
     mark(8);
     if (err == cudaSuccess && on_block) err = (*on_block)(c0, cols);
+    c0 += cols;
   }
 
   hs.k_slab = static_cast<int>(std::min<int64_t>(kKSlabMerged, L.k_pad));
@@ -561,8 +570,54 @@ static int run_stages(int64_t m, int64_t n, int64_t k, const double* A, int64_t 
 int oz2_dgemm_ex(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, const double* B, int64_t ldb,
                  double* C, int64_t ldc, int num_moduli, int quant, int scale, unsigned flags, void* workspace,
                  size_t ws_bytes, void* stream) {
-  return run_stages(m, n, k, A, lda, B, ldb, C, ldc, num_moduli, quant, scale, flags, workspace, ws_bytes, stream, 0,
-                    nullptr);
+  return run_stages(m, n, k, A, lda, B, ldb, C, ldc, num_moduli, quant, scale, flags, workspace, ws_bytes, stream,
+                    nullptr, nullptr);
+}
+
+// Column blocks for oz2_dgemm_host.  C's copy back overlaps the blocks after
+// the one copied, so the last block's copy is exposed: it is one 256-column
+// tile column.  The others take c tile columns each, c from the smallest
+// width that stays within the block budget up to three more, chosen so that
+// the residue GEMM's units (⌈m/256⌉·r per tile column) fill the last wave
+// over its persistent CTA pairs as fully as possible.  Narrow C (n < 1536)
+// is one block.
+static ColumnBlocks host_column_blocks(int64_t m, int64_t n, int r) {
+  ColumnBlocks b;
+  const int64_t tiles = (n + 255) / 256;
+  if (n < 1536 || tiles < 4) {
+    b.count = 1;
+    b.widths[0] = n;
+    return b;
+  }
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int64_t pairs = std::max(1, sms / 2);
+  const int64_t per_tile = (m + 255) / 256 * r;
+  int64_t left = tiles - 1;  // tile columns before the last
+  while (left > 0) {
+    const int64_t slots = kHostBlocksMax - 1 - b.count;  // blocks left before the last one
+    int64_t best_c = left;
+    if (slots > 1) {
+      const int64_t c_min = std::max<int64_t>(3, (left + slots - 1) / slots);
+      double best_idle = 2.0;
+      best_c = std::min(left, c_min);
+      for (int64_t c = c_min; c < c_min + 4 && c <= left; ++c) {
+        const int64_t rest = left - c;
+        if (rest != 0 && rest < 3 && rest < c_min) continue;  // no sliver before the last block
+        const double waves = static_cast<double>(per_tile * c) / static_cast<double>(pairs);
+        const double idle = (std::ceil(waves) - waves) / std::ceil(waves);  // idle share of the launch
+        if (idle < best_idle - 1e-9) {
+          best_idle = idle;
+          best_c = c;
+        }
+      }
+    }
+    b.widths[b.count++] = best_c * 256;
+    left -= best_c;
+  }
+  b.widths[b.count++] = n - 256 * (tiles - 1);  // the last (possibly ragged) tile column
+  return b;
 }
 
 int oz2_dgemm(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, const double* B, int64_t ldb,
@@ -623,8 +678,7 @@ int oz2_dgemm_host(int64_t m, int64_t n, int64_t k, const double* hA, int64_t ld
   // C goes back by column blocks on the copy stream, each as soon as its
   // reconstruction and fallback are done, so that the copies overlap the
   // residue GEMM of the blocks after it.
-  const int64_t nblk = std::max<int64_t>(1, std::min<int64_t>(kHostBlocksMax, (n + kHostBlockCols / 2) / kHostBlockCols));
-  const int64_t col_block = ((n + nblk - 1) / nblk + 255) / 256 * 256;
+  const ColumnBlocks blocks = host_column_blocks(m, n, num_moduli);
   int blk = 0;
   const BlockDone copy_back = [&](int64_t c0, int64_t cols) -> cudaError_t {
     cudaError_t e = cudaEventRecord(ds->block_done[blk], s);
@@ -636,7 +690,7 @@ int oz2_dgemm_host(int64_t m, int64_t n, int64_t k, const double* hA, int64_t ld
   if (err == cudaSuccess) {
     if (k > 0) {
       st = run_stages(m, n, k, dA, m, dB, k, dC, m, num_moduli, OZ2_QUANT_TZ, OZ2_SCALE_R2, 0,
-                      buf + bA + bB + bC, ws, stream, col_block, &copy_back);
+                      buf + bA + bB + bC, ws, stream, &blocks, &copy_back);
     } else {  // C = 0
       err = cudaMemsetAsync(dC, 0, sizeof(double) * m * n, s);
       if (err == cudaSuccess) err = copy_back(0, n);
