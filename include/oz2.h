@@ -109,7 +109,8 @@ int oz2_dgemm(int64_t m, int64_t n, int64_t k,
  * library's memory pool.  A contiguous matrix (ld = rows) moves in one
  * linear copy, any other in a pitched copy.  For wide C (n ≥ 1536) the
  * residue GEMM, reconstruction and fallback run by column blocks (a last
- * block of 256 columns, the others 768 to 1536 wide), and each block of C
+ * block of 256 columns; at most 8 blocks, the others multiples of 256 wide
+ * chosen to fill the GEMM's last wave), and each block of C
  * is copied back on a library-owned copy stream while the next block is
  * computed; the result is the same as unblocked.  Host-buffer calls on one
  * device share that stream and are serialised. */
