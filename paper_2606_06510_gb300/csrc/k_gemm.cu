@@ -88,6 +88,18 @@ __device__ __forceinline__ float combine_residue_short(float a0, float a1, bool 
   const float v = square ? fmaf(s, a1, a0) : fmaf(16.f, a0, -15.f * a1);
   return centred_small(loose_mod(v, m, inv_m), m, inv_m, hi);
 }
+// The short-K kernel's form (k ≤ 128, one k-block): loose_mod leaves r with
+// |r| < 1.5m, so one step toward the centred range [hi + 1 - m, hi] finishes
+// (above hi, r - m ≥ hi + 1 - m; below it, r + m ≤ hi), and SQUARE, uniform
+// over a unit, is a template parameter.
+template <bool SQUARE>
+__device__ __forceinline__ float combine_residue_short1(float a0, float a1, float s, float m, float inv_m,
+                                                        float hi) {
+  const float v = SQUARE ? fmaf(s, a1, a0) : fmaf(16.f, a0, -15.f * a1);
+  float r = loose_mod(v, m, inv_m);
+  r = r > hi ? r - m : r;
+  return r < hi + 1.f - m ? r + m : r;
+}
 // int16 encoding of an integer-valued float in [-2^15, 2^15).
 __device__ __forceinline__ uint32_t as_i16_bits(float r) { return __float_as_uint(r + kRoundMagic) & 0xFFFFu; }
 
@@ -126,7 +138,9 @@ __device__ __forceinline__ int64_t slab_steps_of(const Oz2Moduli& mods, int i, i
 }
 
 // MODE 0: residue planes (all moduli); MODE 1: magnitude planes ("+1" pass).
-template <int MODE>
+// SHORT1: the instance for k ≤ 128 (one k-block, so one short slab for every
+// modulus), whose epilogue takes the single-correction reduction.
+template <int MODE, bool SHORT1 = false>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     plane_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                       const __grid_constant__ Oz2Moduli mods, int64_t k_pad, UnitMap um, EpiCtx ctx) {
@@ -362,7 +376,23 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
             const int64_t cc = col0 + c;
             int16_t* dst = rrow + cc * ctx.ldr;
             const int ncol = ctx.n - cc < 16 ? static_cast<int>(ctx.n - cc) : 16;
-            if (ncol == 16 && short_slab) {  // a single short slab
+            if (SHORT1 && ncol == 16 && square) {  // k ≤ 128: one short slab, every modulus
+#pragma unroll
+              for (int j = 0; j < 16; ++j) {
+                const float rj =
+                    combine_residue_short1<true>(__uint_as_float(v0[j]), __uint_as_float(v1[j]), sb, mf, inv, hi);
+                *dst = static_cast<int16_t>(as_i16_bits(rj));
+                dst += ctx.ldr;
+              }
+            } else if (SHORT1 && ncol == 16) {
+#pragma unroll
+              for (int j = 0; j < 16; ++j) {
+                const float rj =
+                    combine_residue_short1<false>(__uint_as_float(v0[j]), __uint_as_float(v1[j]), sb, mf, inv, hi);
+                *dst = static_cast<int16_t>(as_i16_bits(rj));
+                dst += ctx.ldr;
+              }
+            } else if (!SHORT1 && ncol == 16 && short_slab) {  // a single short slab
 #pragma unroll
               for (int j = 0; j < 16; ++j) {
                 const float rj =
@@ -563,7 +593,7 @@ cudaError_t launch_plane_gemm(int64_t m, int64_t n, int64_t k_pad, const Oz2Modu
   um.ntiles = um.ntm * um.ntn;
   um.nunits = um.ntiles * (mode == 0 ? mods.r : 1);
   const size_t smem = gemm_smem_bytes();
-  auto kern = mode == 0 ? plane_gemm_kernel<0> : plane_gemm_kernel<1>;
+  auto kern = mode == 1 ? plane_gemm_kernel<1> : k_pad == kBK ? plane_gemm_kernel<0, true> : plane_gemm_kernel<0>;
   cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (err != cudaSuccess) return err;
   // Persistent grid: as many CTA pairs as can be resident at once.
