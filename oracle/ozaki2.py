@@ -18,13 +18,15 @@ All You Need (Part 1)") and is written to be checked against it by eye:
   carry-corrected base-16 split, and Eq. (accum-exact).
 * Algorithm 1 and §2.6 contract item (vi): native-FP64 fallback rows.
 
-Where the paper is silent, this module takes the following readings (each is
-repeated in DESIGN.md):
+Where the paper is silent, this module takes the following readings (the
+CUDA path applies the same ones):
 
 R-scale  The "+1" pass computes U = ÂB̂ from power-of-two magnitude planes
          (defined in :func:`magnitude_exponents`); the row/column exponents
-         are then chosen so that Σ_l |Ã_il||B̃_lj| ≤ 2^T with
-         T = ⌊log2 M⌋ - 2 (TZ) or ⌊log2 M⌋ - 4 (RN).  The literal crude bound
+         are then chosen so that Σ_l |Ã_il||B̃_lj| ≤ 2^T, where under TZ
+         T is the largest integer with 2^(T+1) < M (⌊log2 M⌋ - 1 for the
+         products of the moduli used here, none a power of two) and under
+         RN two less.  The literal crude bound
          μ = k·max|Ã|·max|B̃| of Algorithm 1 is kept as scale mode "R1".
 R-moduli r ≤ 12 takes the prefix of S in the order the paper lists it;
          r = 13..16 appends the primes 479, 467, 463, 461.
