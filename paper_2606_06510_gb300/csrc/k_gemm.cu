@@ -4,6 +4,10 @@
 //
 // Work unit = (modulus, 256×256 output tile); units are taken modulus-major
 // so that the planes of one modulus stay in L2 while every pair works on it.
+// The nonsquare moduli, whose units load three stage pairs per k-block
+// against two for a square modulus, come first, and successive waves of
+// units are dealt to the pairs in alternating directions, so that the pairs
+// that take a heavy unit in one wave take a light one in the next.
 // A pair (cluster of 2 CTAs) computes its tile with cta_group::2 MMAs of
 // M = N = 256, K = 32: each CTA holds 128 rows of the A plane tile and 128
 // rows of the B plane tile in its own shared memory, and 128 rows × 256
@@ -112,12 +116,16 @@ struct EpiCtx {
 
 struct UnitMap {
   int64_t ntm, ntn, ntiles, nunits;
+  int nsq, nheavy;  // leading square moduli; nonsquare moduli after them
 };
 
-// Unit u → modulus and tile (grouped raster of kGroupM tile rows).
+// Unit u → modulus and tile (grouped raster of kGroupM tile rows).  Modulus
+// block j of the units is modulus nsq + j for the nheavy nonsquare moduli,
+// then modulus j - nheavy for the squares.
 __device__ __forceinline__ void unit_coords(int64_t u, const UnitMap& um, int* modulus, int64_t* tm, int64_t* tn) {
-  *modulus = static_cast<int>(u / um.ntiles);
-  const int64_t t = u - static_cast<int64_t>(*modulus) * um.ntiles;
+  const int j = static_cast<int>(u / um.ntiles);
+  *modulus = j < um.nheavy ? um.nsq + j : j - um.nheavy;
+  const int64_t t = u - static_cast<int64_t>(j) * um.ntiles;
   const int64_t per_group = kGroupM * um.ntn;
   const int64_t g = t / per_group;
   const int64_t first = g * kGroupM;
@@ -125,6 +133,12 @@ __device__ __forceinline__ void unit_coords(int64_t u, const UnitMap& um, int* m
   const int64_t local = t - g * per_group;
   *tm = first + local % gm;
   *tn = local / gm;
+}
+
+// The unit a pair takes in wave w: waves of npairs units, dealt to the pairs
+// in ascending order in even waves and descending order in odd ones.
+__device__ __forceinline__ int64_t wave_unit(int64_t pair, int64_t w, int64_t npairs) {
+  return w * npairs + ((w & 1) ? npairs - 1 - pair : pair);
 }
 
 template <int MODE>
@@ -186,7 +200,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     if (lane == 0) {
       uint32_t it = 0;
       const uint32_t full_leader0 = mapa_shared(full0, 0);
-      for (int64_t u = pair; u < um.nunits && ok; u += npairs) {
+      for (int64_t w = 0, u = pair; u < um.nunits && ok; u = wave_unit(pair, ++w, npairs)) {
         int i;
         int64_t tm, tn;
         unit_coords(u, um, &i, &tm, &tn);
@@ -243,7 +257,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           p_ ^= 1;
         }
       };
-      for (int64_t u = pair; u < um.nunits && ok; u += npairs) {
+      for (int64_t w = 0, u = pair; u < um.nunits && ok; u = wave_unit(pair, ++w, npairs)) {
         int i;
         int64_t tm, tn;
         unit_coords(u, um, &i, &tm, &tn);
@@ -320,7 +334,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     const uint32_t lane_addr = tmem + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(64 * h);
     const uint32_t acc_empty_leader = mapa_shared(acc_empty, 0);
     uint32_t accph = 0;
-    for (int64_t u = pair; u < um.nunits && ok; u += npairs) {
+    for (int64_t w = 0, u = pair; u < um.nunits && ok; u = wave_unit(pair, ++w, npairs)) {
       int i;
       int64_t tm, tn;
       unit_coords(u, um, &i, &tm, &tn);
@@ -592,6 +606,12 @@ cudaError_t launch_plane_gemm(int64_t m, int64_t n, int64_t k_pad, const Oz2Modu
   um.ntn = (n + kTileN - 1) / kTileN;
   um.ntiles = um.ntm * um.ntn;
   um.nunits = um.ntiles * (mode == 0 ? mods.r : 1);
+  // Square moduli lead the set; the nonsquare ones are scheduled first.
+  um.nsq = 0;
+  while (um.nsq < mods.r && mods.sq_base[um.nsq]) ++um.nsq;
+  um.nheavy = mode == 0 ? mods.r - um.nsq : 0;
+  for (int i = um.nsq; i < mods.r; ++i)
+    if (mods.sq_base[i]) um.nheavy = 0;  // not a prefix: keep the index order
   const size_t smem = gemm_smem_bytes();
   auto kern = mode == 1 ? plane_gemm_kernel<1> : k_pad == kBK ? plane_gemm_kernel<0, true> : plane_gemm_kernel<0>;
   cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
