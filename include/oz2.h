@@ -162,7 +162,10 @@ int oz2_dgemm_ex(int64_t m, int64_t n, int64_t k,
  *   d[m], e[n]            int32  the scale exponents (D = diag 2^d_i ...)
  *   urow[m]               float  max_j U_ij of the "+1" GEMM (R2)
  *   mag_a, mag_b          uint8  magnitude planes Â (m×k_pad), B̂ (n×k_pad),
- *                                row-major
+ *                                row-major.  When the residue GEMM splits K
+ *                                (a small C with a long k) this region is
+ *                                then reused for the partial residues, so
+ *                                after such a call it holds those instead.
  *   planes_a, planes_b    uint8  E4M3 digit planes, see oz2_plane_layout
  *   residues              int16  r matrices C^(i), each m×n column-major
  *                                with ld = res_ld (matrix i starts at element

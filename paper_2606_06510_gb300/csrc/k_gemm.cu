@@ -114,25 +114,57 @@ struct EpiCtx {
   int64_t m, n, ldr;
 };
 
+// Units: (modulus, part of the k-blocks, tile).  With kparts > 1 (split K)
+// each unit covers kpart_steps consecutive k-blocks (the last part fewer)
+// and the epilogue stores its residue as part `part` of the partial-residue
+// planes, which fold_parts_kernel then sums mod m (Eq. modgemm is a sum over
+// k, so C^(i) is the sum of the parts' residues mod m_i).
 struct UnitMap {
   int64_t ntm, ntn, ntiles, nunits;
   int nsq, nheavy;  // leading square moduli; nonsquare moduli after them
+  int64_t ksteps, kparts, kpart_steps;
 };
 
-// Unit u → modulus and tile (grouped raster of kGroupM tile rows).  Modulus
-// block j of the units is modulus nsq + j for the nheavy nonsquare moduli,
-// then modulus j - nheavy for the squares.
-__device__ __forceinline__ void unit_coords(int64_t u, const UnitMap& um, int* modulus, int64_t* tm, int64_t* tn) {
-  const int j = static_cast<int>(u / um.ntiles);
-  *modulus = j < um.nheavy ? um.nsq + j : j - um.nheavy;
-  const int64_t t = u - static_cast<int64_t>(j) * um.ntiles;
+struct Unit {
+  int i, part;         // modulus, part of the k-blocks
+  int64_t tm, tn;      // tile
+  int64_t k_lo, k_hi;  // k-blocks [k_lo, k_hi)
+};
+
+// Unit u (grouped raster of kGroupM tile rows).  Modulus block j of the
+// units is modulus nsq + j for the nheavy nonsquare moduli, then modulus
+// j - nheavy for the squares; within a modulus the parts come in order.
+// The magnitude GEMM (MODE 1) has one modulus and never splits K.
+template <int MODE>
+__device__ __forceinline__ Unit unit_at(int64_t u, const UnitMap& um) {
+  Unit x;
+  int64_t t = u;
+  if (MODE == 1) {
+    x.i = 0;
+    x.part = 0;
+  } else {
+    const int64_t per_mod = um.ntiles * um.kparts;
+    const int j = static_cast<int>(u / per_mod);
+    x.i = j < um.nheavy ? um.nsq + j : j - um.nheavy;
+    const int64_t v = u - static_cast<int64_t>(j) * per_mod;
+    x.part = static_cast<int>(v / um.ntiles);
+    t = v - static_cast<int64_t>(x.part) * um.ntiles;
+  }
   const int64_t per_group = kGroupM * um.ntn;
   const int64_t g = t / per_group;
   const int64_t first = g * kGroupM;
   const int64_t gm = um.ntm - first < kGroupM ? um.ntm - first : kGroupM;
   const int64_t local = t - g * per_group;
-  *tm = first + local % gm;
-  *tn = local / gm;
+  x.tm = first + local % gm;
+  x.tn = local / gm;
+  if (MODE == 1) {
+    x.k_lo = 0;
+    x.k_hi = um.ksteps;
+  } else {
+    x.k_lo = static_cast<int64_t>(x.part) * um.kpart_steps;
+    x.k_hi = um.ksteps - x.k_lo < um.kpart_steps ? um.ksteps : x.k_lo + um.kpart_steps;
+  }
+  return x;
 }
 
 // The unit a pair takes in wave w: waves of npairs units, dealt to the pairs
@@ -201,9 +233,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       uint32_t it = 0;
       const uint32_t full_leader0 = mapa_shared(full0, 0);
       for (int64_t w = 0, u = pair; u < um.nunits && ok; u = wave_unit(pair, ++w, npairs)) {
-        int i;
-        int64_t tm, tn;
-        unit_coords(u, um, &i, &tm, &tn);
+        const Unit x = unit_at<MODE>(u, um);
+        const int i = x.i;
+        const int64_t tm = x.tm, tn = x.tn;
         const int np = planes_of<MODE>(mods, i);
         const int pbase = MODE == 0 ? mods.plane_off[i] : 0;
         const int ya = static_cast<int>(tm * kTileM + rank * kRows);
@@ -213,7 +245,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         // operand's last one lies past the end of the tensor (zero fill).
         const int64_t blk_a = (static_cast<int64_t>(ya / kPlaneRows) * ksteps * mods.nplanes + pbase) * kPlaneRows;
         const int64_t blk_b = (static_cast<int64_t>(yb / kPlaneRows) * ksteps * mods.nplanes + pbase) * kPlaneRows;
-        for (int64_t kb = 0; kb < ksteps && ok; ++kb) {
+        for (int64_t kb = x.k_lo; kb < x.k_hi && ok; ++kb) {
           for (int p = 0; p < np; ++p, ++it) {
             const int s = it % kStages;
             if (!mbar_wait_bounded(empty0 + 8 * s, ((it / kStages) & 1) ^ 1, kWaitLimit)) {
@@ -258,20 +290,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         }
       };
       for (int64_t w = 0, u = pair; u < um.nunits && ok; u = wave_unit(pair, ++w, npairs)) {
-        int i;
-        int64_t tm, tn;
-        unit_coords(u, um, &i, &tm, &tn);
+        const Unit x = unit_at<MODE>(u, um);
+        const int i = x.i;
         const int np = planes_of<MODE>(mods, i);
         const int64_t slab = slab_steps_of<MODE>(mods, i, ksteps);
-        for (int64_t kb0 = 0; kb0 < ksteps && ok; kb0 += slab) {
+        for (int64_t kb0 = x.k_lo; kb0 < x.k_hi && ok; kb0 += slab) {
           if (!mbar_wait_bounded(acc_empty, accph ^ 1, kWaitLimit)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const int64_t kb1 = min(ksteps, kb0 + slab);
+          const int64_t kb1 = min(x.k_hi, kb0 + slab);
           for (int64_t kb = kb0; kb < kb1 && ok; ++kb) {
-            const uint32_t first = kb == 0 ? 0u : 1u;  // later slabs add to the carried residue
+            const uint32_t first = kb == x.k_lo ? 0u : 1u;  // later slabs add to the carried residue
             if (np == 2) {  // square: stages (d0,e0) and (d1,e1)
               uint32_t s1 = st, p1 = ph;
               next(s1, p1);
@@ -335,9 +366,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     const uint32_t acc_empty_leader = mapa_shared(acc_empty, 0);
     uint32_t accph = 0;
     for (int64_t w = 0, u = pair; u < um.nunits && ok; u = wave_unit(pair, ++w, npairs)) {
-      int i;
-      int64_t tm, tn;
-      unit_coords(u, um, &i, &tm, &tn);
+      const Unit x = unit_at<MODE>(u, um);
+      const int i = x.i;
+      const int64_t tm = x.tm, tn = x.tn;
       const int64_t row = tm * kTileM + rank * kRows + 32 * q + lane;
       const int64_t col0 = tn * kTileN + 64 * h;
       const bool square = MODE == 0 ? mods.sq_base[i] != 0 : true;
@@ -345,18 +376,20 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       const float inv = 1.f / mf;
       const float sb = MODE == 0 ? static_cast<float>(mods.sq_base[i]) : 0.f;
       const float hi = MODE == 0 ? static_cast<float>(mods.m[i] - 1 - mods.m[i] / 2) : 0.f;
-      // This thread's row of C^(i); column j at rrow[j·ldr] (a warp stores 32
-      // consecutive rows of one column, 64 contiguous bytes, per instruction).
-      int16_t* rrow = MODE == 0 ? ctx.res + static_cast<size_t>(i) * ctx.n * ctx.ldr + row : nullptr;
+      // This thread's row of C^(i) (of part `part` of it under split K);
+      // column j at rrow[j·ldr] (a warp stores 32 consecutive rows of one
+      // column, 64 contiguous bytes, per instruction).
+      int16_t* rrow =
+          MODE == 0 ? ctx.res + (static_cast<size_t>(x.part) * mods.r + i) * ctx.n * ctx.ldr + row : nullptr;
       const int64_t slab = slab_steps_of<MODE>(mods, i, ksteps);
-      // Short slabs (K = 128·ksteps k-entries): v stays an integer below 2^24
+      // Short slabs (K = 128·(k_hi - k_lo) k-entries): v stays an integer below 2^24
       // without reducing the accumulators first.  Square moduli (|d0e0| ≤ 256,
       // |d1e0 + d0e1| ≤ 512, s ≤ 33): |v| ≤ K(256 + 33·512) < 2^24 for K ≤ 896.
       // Nonsquare (|(d0+d1)(e0+e1)| ≤ 22², merged term ≤ 4095):
       // |16·acc0 - 15·acc1| ≤ K(16·484 + 15·4095) < 2^24 for K ≤ 128.
-      const bool short_slab = MODE == 0 && ksteps <= (square ? 7 : 1);
+      const bool short_slab = MODE == 0 && x.k_hi - x.k_lo <= (square ? 7 : 1);
       float rowmax = 0.f;
-      for (int64_t kb0 = 0; kb0 < ksteps; kb0 += slab) {
+      for (int64_t kb0 = x.k_lo; kb0 < x.k_hi; kb0 += slab) {
         if (!mbar_wait_bounded(acc_full, accph, kWaitLimit)) {
           ok = false;
           break;
@@ -367,7 +400,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         // acc1 = 0 for square moduli (v = acc0 + s·acc1), and acc0 = acc1 = r
         // for nonsquare ones (16r - 15r = r).  The bounds of Eq. accum-exact
         // keep their margin: 32768·256 + 544 and 4096·4095 + 255 < 2^24.
-        const bool carry = MODE == 0 && kb0 + slab < ksteps;
+        const bool carry = MODE == 0 && kb0 + slab < x.k_hi;
         for (int c = 0; c < 64; c += 16) {
           uint32_t v0[16], v1[16];
           tmem_ld16(lane_addr + c, v0);
@@ -573,6 +606,120 @@ static bool make_block_map(CUtensorMap* map, const uint8_t* base, int64_t rows, 
   return r == CUDA_SUCCESS;
 }
 
+// ---------------------------------------------------------------------------
+// Split K.  A problem whose units fill few waves of the CTA pairs (a small C
+// with a long k) runs each unit's k-blocks in kparts parts; the parts'
+// residues land in scratch planes [part][modulus][column][row] and
+// fold_parts_kernel sums them mod m into C^(i).
+// ---------------------------------------------------------------------------
+constexpr int kFoldThreads = 128;
+
+// C^(i) from its parts: the sum of kparts centred residues has magnitude at
+// most kparts·⌊m/2⌋ < 2^16, so centred_small reduces it exactly.  One thread
+// takes 8 consecutive rows of one column (16-byte loads: ldr is a multiple
+// of 8 and both buffers are 16-byte aligned); blockIdx.z is the modulus.
+__global__ void __launch_bounds__(kFoldThreads) fold_parts_kernel(const int16_t* __restrict__ part,
+                                                                  int16_t* __restrict__ res, int64_t m, int64_t n,
+                                                                  int64_t ldr, int kparts,
+                                                                  const __grid_constant__ Oz2Moduli mods) {
+  const int i = blockIdx.z;
+  const float mf = static_cast<float>(mods.m[i]), inv = 1.f / mf;
+  const float hi = static_cast<float>(mods.m[i] - 1 - mods.m[i] / 2);
+  const int64_t row0 = (static_cast<int64_t>(blockIdx.x) * kFoldThreads + threadIdx.x) * 8;
+  if (row0 >= m) return;
+  const size_t plane = static_cast<size_t>(n) * ldr, pstride = static_cast<size_t>(mods.r) * plane;
+  for (int64_t col = blockIdx.y; col < n; col += gridDim.y) {
+    const size_t off = static_cast<size_t>(i) * plane + static_cast<size_t>(col) * ldr + row0;
+    if (row0 + 8 <= m) {
+      int acc[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) acc[j] = 0;
+      for (int p = 0; p < kparts; ++p) {
+        const uint4 v = __ldg(reinterpret_cast<const uint4*>(part + p * pstride + off));
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          acc[2 * j] += static_cast<int16_t>(w[j] & 0xFFFFu);
+          acc[2 * j + 1] += static_cast<int>(w[j]) >> 16;
+        }
+      }
+      uint32_t o[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        o[j] = as_i16_bits(centred_small(static_cast<float>(acc[2 * j]), mf, inv, hi)) |
+               (as_i16_bits(centred_small(static_cast<float>(acc[2 * j + 1]), mf, inv, hi)) << 16);
+      *reinterpret_cast<uint4*>(res + off) = make_uint4(o[0], o[1], o[2], o[3]);
+    } else {
+      for (int64_t r = row0; r < m; ++r) {
+        int a = 0;
+        for (int p = 0; p < kparts; ++p) a += part[p * pstride + off + (r - row0)];
+        res[off + (r - row0)] = static_cast<int16_t>(as_i16_bits(centred_small(static_cast<float>(a), mf, inv, hi)));
+      }
+    }
+  }
+}
+
+constexpr int64_t kMaxKParts = 16;     // keeps kparts·⌊m/2⌋ < 2^16 for the fold
+constexpr int64_t kMinPartSteps = 4;   // k-blocks (512 k-entries) per part at least
+
+// Estimated duration of the residue GEMM under the unit schedule (nonsquare
+// moduli first, waves dealt in alternating directions), in units of one
+// stage pair on a CTA pair (a 256×256×128 FP8 product, about 0.39 µs at
+// 2.07 GHz): the largest load over the pairs.  A nonsquare unit of s
+// k-blocks costs 3s plus 10 per epilogue drain (one per 4096 k-entries), a
+// square one 2s plus 10 per 32768.  A split adds the fold (its bytes at
+// about 5 TB/s, and a launch).  The pairs' loads are piecewise constant in
+// the pair index, changing only where the heavy units and all units end in
+// their last waves, so those pairs and the two ends cover the maximum.
+static double split_cost(int64_t ntiles, int r, int nsq, int64_t ksteps, int64_t kparts, int64_t pairs, int64_t m,
+                         int64_t n) {
+  const int64_t s = (ksteps + kparts - 1) / kparts;
+  const int64_t U = ntiles * r * kparts, H = ntiles * (r - nsq) * kparts;
+  const int64_t P = std::max<int64_t>(1, std::min(pairs, U));
+  constexpr int64_t kSlabM = kKSlabMerged / kBK, kSlabS = kKSlabSquare / kBK;
+  const double wh = 3.0 * s + 10.0 * ((s + kSlabM - 1) / kSlabM);
+  const double wl = 2.0 * s + 10.0 * ((s + kSlabS - 1) / kSlabS);
+  auto count = [&](int64_t X, int64_t q) {  // units below X that pair q takes
+    const int64_t w0 = X / P, rem = X - w0 * P;
+    const int64_t pos = (w0 & 1) ? P - 1 - q : q;
+    return w0 + (pos < rem ? 1 : 0);
+  };
+  auto load = [&](int64_t q) {
+    const int64_t h = count(H, q);
+    return h * wh + (count(U, q) - h) * wl;
+  };
+  double mx = std::max(load(0), load(P - 1));
+  for (const int64_t X : {H, U}) {
+    const int64_t w0 = X / P, rem = X - w0 * P;
+    const int64_t b = (w0 & 1) ? P - rem : rem;
+    for (const int64_t q : {b - 1, b})
+      if (q >= 0 && q < P) mx = std::max(mx, load(q));
+  }
+  if (kparts > 1) mx += (3.0 + (kparts + 1.0) * r * m * n * 2.0 / 5.0e6) / 0.39;
+  return mx;
+}
+
+// Parts of K per residue-GEMM unit: 1 unless the units fill fewer than four
+// waves and a split of at most max_parts (each part non-empty and at least
+// kMinPartSteps k-blocks) is estimated at least 5% faster.
+static int64_t choose_kparts(int64_t ntiles, int r, int nsq, int64_t ksteps, int64_t pairs, int64_t m, int64_t n,
+                             int64_t max_parts) {
+  if (max_parts < 2 || ntiles * r >= 4 * pairs) return 1;
+  int64_t best = 1;
+  double best_cost = split_cost(ntiles, r, nsq, ksteps, 1, pairs, m, n);
+  for (int64_t p = 2; p <= max_parts; ++p) {
+    const int64_t s = (ksteps + p - 1) / p;
+    if (s < kMinPartSteps) break;
+    if ((ksteps + s - 1) / s != p) continue;  // a part would be empty
+    const double c = split_cost(ntiles, r, nsq, ksteps, p, pairs, m, n);
+    if (c < 0.95 * best_cost) {
+      best = p;
+      best_cost = c;
+    }
+  }
+  return best;
+}
+
 static size_t gemm_smem_bytes() { return 1024 + static_cast<size_t>(kStages) * kStageBytes + 8 * (2 * kStages + 3); }
 
 static int num_sms() {
@@ -586,7 +733,8 @@ static int num_sms() {
 //       2 residues (SIMT reference), 3 magnitude (SIMT reference).
 cudaError_t launch_plane_gemm(int64_t m, int64_t n, int64_t k_pad, const Oz2Moduli& mods,
                               const uint8_t* planes_a, const uint8_t* planes_b, int mode,
-                              int16_t* residues, int64_t ldr, float* urow, Oz2Device* dev, cudaStream_t st) {
+                              int16_t* residues, int64_t ldr, float* urow, Oz2Device* dev, cudaStream_t st,
+                              int16_t* partials, size_t partial_bytes) {
   if (m == 0 || n == 0) return cudaSuccess;
   EpiCtx ctx{residues, urow, dev, m, n, ldr};
   if (mode >= 2) {
@@ -612,6 +760,9 @@ cudaError_t launch_plane_gemm(int64_t m, int64_t n, int64_t k_pad, const Oz2Modu
   um.nheavy = mode == 0 ? mods.r - um.nsq : 0;
   for (int i = um.nsq; i < mods.r; ++i)
     if (mods.sq_base[i]) um.nheavy = 0;  // not a prefix: keep the index order
+  um.ksteps = k_pad / kBK;
+  um.kparts = 1;
+  um.kpart_steps = um.ksteps;
   const size_t smem = gemm_smem_bytes();
   auto kern = mode == 1 ? plane_gemm_kernel<1> : k_pad == kBK ? plane_gemm_kernel<0, true> : plane_gemm_kernel<0>;
   cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
@@ -636,9 +787,28 @@ cudaError_t launch_plane_gemm(int64_t m, int64_t n, int64_t k_pad, const Oz2Modu
     else
       cudaGetLastError();
   }
+  // Split K where the scratch holds the parts (16-byte aligned rows: the
+  // fold reads and writes 8 residues at a time).
+  if (mode == 0 && partials && ldr % 8 == 0 && reinterpret_cast<uintptr_t>(partials) % 16 == 0 &&
+      reinterpret_cast<uintptr_t>(residues) % 16 == 0) {
+    const size_t part_bytes = static_cast<size_t>(mods.r) * n * ldr * sizeof(int16_t);
+    const int64_t max_parts = std::min<int64_t>(kMaxKParts, static_cast<int64_t>(partial_bytes / part_bytes));
+    const int nheavy_sq = um.nheavy ? um.nsq : mods.r;  // the model's squares
+    um.kparts = choose_kparts(um.ntiles, mods.r, nheavy_sq, um.ksteps, pairs, m, n, max_parts);
+    um.kpart_steps = (um.ksteps + um.kparts - 1) / um.kparts;
+    um.nunits *= um.kparts;
+    if (um.kparts > 1) ctx.res = partials;
+  }
   pairs = std::max<int64_t>(1, std::min<int64_t>(pairs, um.nunits));
   count_launch();
   kern<<<static_cast<unsigned>(2 * pairs), kGemmThreads, smem, st>>>(ta, tb, mods, k_pad, um, ctx);
+  if (um.kparts > 1) {
+    const int64_t row_threads = (m + 7) / 8;
+    dim3 g(static_cast<unsigned>((row_threads + kFoldThreads - 1) / kFoldThreads),
+           static_cast<unsigned>(std::min<int64_t>(n, 32768)), static_cast<unsigned>(mods.r));
+    count_launch();
+    fold_parts_kernel<<<g, kFoldThreads, 0, st>>>(partials, residues, m, n, ldr, static_cast<int>(um.kparts), mods);
+  }
   return cudaGetLastError();
 }
 

@@ -550,7 +550,10 @@ static int run_stages(int64_t m, int64_t n, int64_t k, const double* A, int64_t 
     const int64_t cols = blocked ? blocks->widths[bi] : n;
     const uint8_t* pb0 = pb + static_cast<size_t>(c0 / kPlaneRows) * (L.k_pad / kPlaneLine) * L.num_planes *
                                   static_cast<size_t>(kPlaneBlock);
-    err = launch_plane_gemm(m, cols, L.k_pad, mods, pa, pb0, simt ? 2 : 0, res, L.res_ld, nullptr, ds->status, s);
+    // The magnitude planes are dead once the scales are chosen: their region
+    // is the scratch for the partial residues of a split-K residue GEMM.
+    err = launch_plane_gemm(m, cols, L.k_pad, mods, pa, pb0, simt ? 2 : 0, res, L.res_ld, nullptr, ds->status, s,
+                            reinterpret_cast<int16_t*>(mag_a), L.planes_a - L.mag_a);
     mark(6);
     if (err == cudaSuccess) err = launch_reconstruct(m, cols, mods, res, L.res_ld, d, e + c0, C + c0 * ldc, ldc, s);
     mark(7);

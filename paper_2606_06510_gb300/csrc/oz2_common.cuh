@@ -419,9 +419,12 @@ cudaError_t launch_deconstruct(int64_t m, int64_t n, int64_t k, const Oz2Moduli&
                                const double* B, int64_t ldb, const int32_t* d, const int32_t* e,
                                const uint8_t* row_flag, const uint8_t* col_flag, int quant,
                                uint8_t* planes_a, uint8_t* planes_b, cudaStream_t st);
+// `partials` (16-byte aligned, `partial_bytes` long, or null) is scratch the
+// residue GEMM may split K into; it must not overlap the operands or C^(i).
 cudaError_t launch_plane_gemm(int64_t m, int64_t n, int64_t k_pad, const Oz2Moduli& mods,
                               const uint8_t* planes_a, const uint8_t* planes_b, int mode,
-                              int16_t* residues, int64_t ldr, float* urow, Oz2Device* dev, cudaStream_t st);
+                              int16_t* residues, int64_t ldr, float* urow, Oz2Device* dev, cudaStream_t st,
+                              int16_t* partials = nullptr, size_t partial_bytes = 0);
 cudaError_t launch_reconstruct(int64_t m, int64_t n, const Oz2Moduli& mods,
                                const int16_t* residues, int64_t ldr, const int32_t* d,
                                const int32_t* e, double* C, int64_t ldc, cudaStream_t st);

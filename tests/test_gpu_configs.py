@@ -96,9 +96,10 @@ def test_gemv_batch16_character(oz):
 
 
 def test_very_long_k_many_slabs(oz):
-    """k = 262144: eight K-slabs for the square moduli and 64 for the merged
-    nonsquare ones, so the partial residue is carried in the accumulators
-    many times over; the "+1" pass clamp is at its small end (c = 3)."""
+    """k = 262144: the residue GEMM splits K into 12 parts of 171 k-blocks,
+    and each part carries its nonsquare moduli's partial residue in the
+    accumulators over six 4096-entry K-slabs; the "+1" pass clamp is at its
+    small end (c = 3)."""
     m, n, k = 9, 7, 262144  # one ragged tile: the slab logic is per tile
     A = np.array(wl.random_matrix(m, k, 0.5, 9300), order="F")
     B = np.array(wl.random_matrix(k, n, 0.5, 9400), order="F")
