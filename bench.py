@@ -43,8 +43,8 @@ GEMM_SOURCE = os.path.join(ROOT, "paper_2606_06510_gb300", "csrc", "k_gemm.cu")
 # DRAM read+write bytes of one residue-GEMM launch, from the ncu capture in
 # profiles/residue_gemm_dgemm_4096.md; reported only while the kernel source
 # is the one the counters were taken on.
-GEMM_TRAFFIC = {"workload": "dgemm_4096", "num_moduli": 12, "bytes": 2.1105e9,
-                "sha256": "8a4ceeae02435a3347028abf7cf856c335e571a4830eeb9400c83a4760555d3f"}
+GEMM_TRAFFIC = {"workload": "dgemm_4096", "num_moduli": 12, "bytes": 2.1354e9,
+                "sha256": "c50e3a3c41231d493c83ef684dd0fc7dc4b492d5c893fe8c18856faf11bbd00b"}
 
 
 def gemm_traffic(w, r):
