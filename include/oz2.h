@@ -182,6 +182,29 @@ typedef struct {
 int oz2_workspace_layout(int64_t m, int64_t n, int64_t k, int num_moduli,
                          oz2_ws_layout* out);
 
+/* How the library runs a problem on a GPU with cta_pairs CTA pairs (half its
+ * SM count: 76 on a GB300).  Host arithmetic only: it touches no device and
+ * runs without one.
+ *   kparts        parts of k per residue-GEMM unit in oz2_dgemm_ex and
+ *                 oz2_dgemm (1: no split).  A small C with a long k fills
+ *                 few waves of the CTA pairs; each unit then covers 1/kparts
+ *                 of the k-blocks, and a fold sums the parts' residues mod m.
+ *   host_blocks   column blocks of oz2_dgemm_host (1 to 8).  The blocks run
+ *                 the residue GEMM, reconstruction and fallback one after
+ *                 another, each copied back while the next computes.
+ *   host_widths   their widths: multiples of 256 but the last, which is
+ *                 the last (possibly ragged) 256-column tile column.
+ *   host_kparts   the residue GEMM's kparts for each block.
+ * Returns OZ2_OK, OZ2_ERR_INVALID_ARG (null out, negative sizes,
+ * cta_pairs < 1) or OZ2_ERR_UNSUPPORTED_R. */
+typedef struct {
+  int64_t kparts;
+  int32_t host_blocks;
+  int64_t host_widths[8];
+  int64_t host_kparts[8];
+} oz2_plan_info;
+int oz2_plan(int64_t m, int64_t n, int64_t k, int num_moduli, int cta_pairs, oz2_plan_info* out);
+
 /* Digit-plane layout (§2.5).  For operand X with `rows` rows (m for A, n
  * for B) there are P planes (the return value), each logically a rows×k_pad
  * byte matrix zero-padded from k to k_pad, stored as 128 × 128-byte blocks

@@ -50,6 +50,11 @@ class oz2_ws_layout(ctypes.Structure):
                [("k_pad", ctypes.c_int64), ("num_planes", ctypes.c_int32), ("res_ld", ctypes.c_int64)]
 
 
+class oz2_plan_info(ctypes.Structure):
+    _fields_ = [("kparts", ctypes.c_int64), ("host_blocks", ctypes.c_int32),
+                ("host_widths", ctypes.c_int64 * 8), ("host_kparts", ctypes.c_int64 * 8)]
+
+
 _I64, _P, _I, _U, _SZ = ctypes.c_int64, ctypes.c_void_p, ctypes.c_int, ctypes.c_uint, ctypes.c_size_t
 _SIGS = {
     "oz2_dgemm": (_I, [_I64, _I64, _I64, _P, _I64, _P, _I64, _P, _I64, _I, _P]),
@@ -59,6 +64,7 @@ _SIGS = {
     "oz2_dgemm_ex": (_I, [_I64, _I64, _I64, _P, _I64, _P, _I64, _P, _I64, _I, _I, _I, _U, _P, _SZ, _P]),
     "oz2_workspace_layout": (_I, [_I64, _I64, _I64, _I, ctypes.POINTER(oz2_ws_layout)]),
     "oz2_plane_layout": (_I, [_I, _P]),
+    "oz2_plan": (_I, [_I64, _I64, _I64, _I, _I, ctypes.POINTER(oz2_plan_info)]),
     "oz2_get_stats": (_I, [ctypes.POINTER(oz2_stats)]),
     "oz2_trim_memory": (_I, []),
     "oz2_selftest_timeout": (_I, [ctypes.c_longlong, _P]),
@@ -172,6 +178,16 @@ def oz2_workspace_layout(m: int, n: int, k: int, num_moduli: int) -> dict:
     L = oz2_ws_layout()
     _check(lib().oz2_workspace_layout(m, n, k, num_moduli, ctypes.byref(L)), "oz2_workspace_layout")
     return {name: getattr(L, name) for name, _ in L._fields_}
+
+
+def oz2_plan(m: int, n: int, k: int, num_moduli: int = 12, cta_pairs: int = 76) -> dict:
+    """How the library runs an m×n×k problem on cta_pairs CTA pairs (host
+    arithmetic only): the residue GEMM's parts of k, and the column blocks
+    of oz2_dgemm_host with each block's parts of k."""
+    P = oz2_plan_info()
+    _check(lib().oz2_plan(m, n, k, num_moduli, cta_pairs, ctypes.byref(P)), "oz2_plan")
+    nb = P.host_blocks
+    return {"kparts": P.kparts, "host_widths": list(P.host_widths[:nb]), "host_kparts": list(P.host_kparts[:nb])}
 
 
 def oz2_plane_layout(num_moduli: int):

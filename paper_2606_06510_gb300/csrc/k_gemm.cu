@@ -720,6 +720,15 @@ static int64_t choose_kparts(int64_t ntiles, int r, int nsq, int64_t ksteps, int
   return best;
 }
 
+int64_t residue_gemm_kparts(int64_t m, int64_t n, int64_t k_pad, int r, int nsq, int64_t ldr, size_t partial_bytes,
+                            int64_t pairs) {
+  if (m <= 0 || n <= 0 || k_pad <= 0 || r < 1 || ldr < m || ldr % 8 != 0 || pairs < 1) return 1;
+  const size_t part_bytes = static_cast<size_t>(r) * n * ldr * sizeof(int16_t);
+  const int64_t max_parts = std::min<int64_t>(kMaxKParts, static_cast<int64_t>(partial_bytes / part_bytes));
+  const int64_t ntiles = ((m + kTileM - 1) / kTileM) * ((n + kTileN - 1) / kTileN);
+  return choose_kparts(ntiles, r, nsq, k_pad / kBK, pairs, m, n, max_parts);
+}
+
 static size_t gemm_smem_bytes() { return 1024 + static_cast<size_t>(kStages) * kStageBytes + 8 * (2 * kStages + 3); }
 
 static int num_sms() {
@@ -789,12 +798,10 @@ cudaError_t launch_plane_gemm(int64_t m, int64_t n, int64_t k_pad, const Oz2Modu
   }
   // Split K where the scratch holds the parts (16-byte aligned rows: the
   // fold reads and writes 8 residues at a time).
-  if (mode == 0 && partials && ldr % 8 == 0 && reinterpret_cast<uintptr_t>(partials) % 16 == 0 &&
+  if (mode == 0 && partials && reinterpret_cast<uintptr_t>(partials) % 16 == 0 &&
       reinterpret_cast<uintptr_t>(residues) % 16 == 0) {
-    const size_t part_bytes = static_cast<size_t>(mods.r) * n * ldr * sizeof(int16_t);
-    const int64_t max_parts = std::min<int64_t>(kMaxKParts, static_cast<int64_t>(partial_bytes / part_bytes));
     const int nheavy_sq = um.nheavy ? um.nsq : mods.r;  // the model's squares
-    um.kparts = choose_kparts(um.ntiles, mods.r, nheavy_sq, um.ksteps, pairs, m, n, max_parts);
+    um.kparts = residue_gemm_kparts(m, n, k_pad, mods.r, nheavy_sq, ldr, partial_bytes, pairs);
     um.kpart_steps = (um.ksteps + um.kparts - 1) / um.kparts;
     um.nunits *= um.kparts;
     if (um.kparts > 1) ctx.res = partials;

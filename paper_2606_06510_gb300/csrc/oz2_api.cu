@@ -438,6 +438,14 @@ size_t oz2_workspace_size(int64_t m, int64_t n, int64_t k, int num_moduli) {
   return L.total;
 }
 
+// Leading square moduli of the first r (the published set lists its squares
+// first); the residue GEMM schedules the nonsquare ones before them.
+static int leading_squares(int r) {
+  int q = 0;
+  while (q < r && isqrt_exact(kModuliAll[q])) ++q;
+  return q;
+}
+
 int oz2_workspace_layout(int64_t m, int64_t n, int64_t k, int num_moduli, oz2_ws_layout* out) {
   if (!out || m < 0 || n < 0 || k < 0) return OZ2_ERR_INVALID_ARG;
   if (num_moduli < 1 || num_moduli > kMaxModuli) return OZ2_ERR_UNSUPPORTED_R;
@@ -584,7 +592,7 @@ int oz2_dgemm_ex(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, 
 // the residue GEMM's units (⌈m/256⌉·r per tile column) fill the last wave
 // over its persistent CTA pairs as fully as possible.  Narrow C (n < 1536)
 // is one block.
-static ColumnBlocks host_column_blocks(int64_t m, int64_t n, int r) {
+static ColumnBlocks host_column_blocks(int64_t m, int64_t n, int r, int64_t pairs) {
   ColumnBlocks b;
   const int64_t tiles = (n + 255) / 256;
   if (n < 1536 || tiles < 4) {
@@ -592,10 +600,6 @@ static ColumnBlocks host_column_blocks(int64_t m, int64_t n, int r) {
     b.widths[0] = n;
     return b;
   }
-  int dev = 0, sms = 148;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  const int64_t pairs = std::max(1, sms / 2);
   const int64_t per_tile = (m + 255) / 256 * r;
   int64_t left = tiles - 1;  // tile columns before the last
   while (left > 0) {
@@ -621,6 +625,28 @@ static ColumnBlocks host_column_blocks(int64_t m, int64_t n, int r) {
   }
   b.widths[b.count++] = n - 256 * (tiles - 1);  // the last (possibly ragged) tile column
   return b;
+}
+
+int oz2_plan(int64_t m, int64_t n, int64_t k, int num_moduli, int cta_pairs, oz2_plan_info* out) {
+  if (!out || m < 0 || n < 0 || k < 0 || cta_pairs < 1) return OZ2_ERR_INVALID_ARG;
+  if (num_moduli < 1 || num_moduli > kMaxModuli) return OZ2_ERR_UNSUPPORTED_R;
+  *out = oz2_plan_info{};
+  oz2_ws_layout L;
+  compute_layout(m, n, k, num_moduli, &L);
+  // The split-K scratch is the magnitude-plane region (dead by then).
+  auto kparts = [&](int64_t cols) -> int64_t {
+    if (m == 0 || cols == 0 || k == 0) return 1;
+    return residue_gemm_kparts(m, cols, L.k_pad, num_moduli, leading_squares(num_moduli), L.res_ld,
+                               L.planes_a - L.mag_a, cta_pairs);
+  };
+  out->kparts = kparts(n);
+  const ColumnBlocks b = host_column_blocks(m, n, num_moduli, cta_pairs);
+  out->host_blocks = b.count;
+  for (int i = 0; i < b.count; ++i) {
+    out->host_widths[i] = b.widths[i];
+    out->host_kparts[i] = kparts(b.widths[i]);
+  }
+  return OZ2_OK;
 }
 
 int oz2_dgemm(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, const double* B, int64_t ldb,
@@ -681,7 +707,10 @@ int oz2_dgemm_host(int64_t m, int64_t n, int64_t k, const double* hA, int64_t ld
   // C goes back by column blocks on the copy stream, each as soon as its
   // reconstruction and fallback are done, so that the copies overlap the
   // residue GEMM of the blocks after it.
-  const ColumnBlocks blocks = host_column_blocks(m, n, num_moduli);
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const ColumnBlocks blocks = host_column_blocks(m, n, num_moduli, std::max(1, sms / 2));
   int blk = 0;
   const BlockDone copy_back = [&](int64_t c0, int64_t cols) -> cudaError_t {
     cudaError_t e = cudaEventRecord(ds->block_done[blk], s);

@@ -419,6 +419,12 @@ cudaError_t launch_deconstruct(int64_t m, int64_t n, int64_t k, const Oz2Moduli&
                                const double* B, int64_t ldb, const int32_t* d, const int32_t* e,
                                const uint8_t* row_flag, const uint8_t* col_flag, int quant,
                                uint8_t* planes_a, uint8_t* planes_b, cudaStream_t st);
+// Parts of K per unit the residue GEMM takes for an m×n C (1: no split),
+// with the r moduli of which the first nsq are squares, residues with
+// leading dimension ldr, partial_bytes of scratch and `pairs` CTA pairs.
+// Host-only arithmetic.
+int64_t residue_gemm_kparts(int64_t m, int64_t n, int64_t k_pad, int r, int nsq, int64_t ldr, size_t partial_bytes,
+                            int64_t pairs);
 // `partials` (16-byte aligned, `partial_bytes` long, or null) is scratch the
 // residue GEMM may split K into; it must not overlap the operands or C^(i).
 cudaError_t launch_plane_gemm(int64_t m, int64_t n, int64_t k_pad, const Oz2Moduli& mods,

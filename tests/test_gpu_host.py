@@ -103,3 +103,19 @@ def test_randomised_wide_problems(oz, seed):
     got = oz.oz2_dgemm_host(A, B, num_moduli=r)
     assert_same(got, want)
     assert oz.oz2_check_device_status() == 0
+
+
+def test_column_blocks_with_split_k(oz):
+    """A short C with a long k: each column block's residue GEMM splits k
+    (blocks of 1536, 1024 and 40 columns in 2, 3 and 6 parts on a GB300),
+    with a fallback row and a zero column."""
+    m, n, k = 64, 2600, 5000
+    plan = oz.oz2_plan(m, n, k, 12)
+    assert plan["host_widths"] == [1536, 1024, 40] and min(plan["host_kparts"]) > 1
+    A = np.array(wl.random_matrix(m, k, 1.0, 7500), order="F")
+    B = np.array(wl.random_matrix(k, n, 1.0, 7600), order="F")
+    A[9, :] *= 2.0 ** -300
+    B[:, 2000] = 0.0
+    got = oz.oz2_dgemm_host(A, B, num_moduli=12)
+    assert_same(got, orc.oz2_dgemm(A, B, 12).C)
+    assert oz.oz2_check_device_status() == 0
