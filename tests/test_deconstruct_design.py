@@ -1,0 +1,172 @@
+"""The deconstruction's 32-bit integer arithmetic against the oracle.
+
+The deconstruction (Algorithm 1, quantise and deconstruct; §2.5) computes
+each entry's centred residues with 32-bit integer steps:
+
+* a branch-free truncating quantisation: the significand shifted up by 10
+  and back down with clamping funnel shifts, the sign applied as a two's
+  complement, for scales d ≤ 1083 (and d = -4096 for rows that are zero);
+* Ã split into three 16-bit limbs and a signed top limb, the lowest biased
+  by 2^25, summed per modulus with the limb weights 2^16j mod m pre-scaled
+  by 4;
+* a multiply-high quotient by ⌈2^30/m⌉ that may be one too large, so the
+  remainder lies in [-4m, 4m) and indexes a table of 2m entries rotated by
+  the bias (nonsquare moduli);
+* for square moduli, an added constant that makes the remainder the centred
+  residue plus ⌊m/2⌋, then balanced base-s digits by a multiply-high.
+
+These CPU tests evaluate those steps with 32-bit wrap-around, with every
+constant recomputed from its definition, and compare them with the oracle's
+quantiser, centred residues and digit functions.
+"""
+import numpy as np
+import pytest
+
+from oracle import ozaki2 as orc
+
+M32 = np.uint64(0xFFFFFFFF)
+BIAS = 1 << 25          # the limb-sum bias
+TZ_FAST_MAX_D = 1083    # largest scale the branch-free path takes
+
+
+def u64(x):
+    return np.asarray(x, dtype=np.uint64)
+
+
+def funnel_right_clamped(lo, hi, sh):
+    """Low word of (hi:lo) >> min(sh, 32)."""
+    s = np.minimum(sh, np.uint64(32))
+    return ((hi << np.uint64(32)) | lo) >> s & M32
+
+
+def quantise_tz_limbs(x, d):
+    """The kernel's limbs (b, u1, u2, u3) of trunc(x·2^d)."""
+    bits = np.asarray(x, dtype=np.float64).view(np.uint64)
+    hi, lo = bits >> np.uint64(32), bits & M32
+    E = ((hi >> np.uint64(20)) & np.uint64(0x7FF)).astype(np.int64)
+    mh = (hi & np.uint64(0xFFFFF)) | np.where(E != 0, np.uint64(0x100000), np.uint64(0))
+    r = u64((10 + 1075 - np.maximum(E, 1) - np.asarray(d, dtype=np.int64)) & 0xFFFFFFFF)
+    ph = ((mh << np.uint64(10)) | (lo >> np.uint64(22))) & M32
+    pl = (lo << np.uint64(10)) & M32
+    wide = r >= np.uint64(32)
+    x1 = np.where(wide, np.uint64(0), ph)
+    x0 = np.where(wide, ph, pl)
+    rr = np.where(wide, r - np.uint64(32), r)
+    al = funnel_right_clamped(x0, x1, rr)
+    ah = funnel_right_clamped(x1, np.uint64(0), rr)
+    neg = (hi >> np.uint64(31)) != 0
+    sgn = np.where(neg, M32, np.uint64(0))
+    t = (((ah ^ sgn) << np.uint64(32)) | (al ^ sgn)) + neg.astype(np.uint64)  # two's complement negation
+    tl = t & M32
+    th = (t >> np.uint64(32)).astype(np.int64)
+    th = np.where(th >= 1 << 31, th - (1 << 32), th)
+    b = ((tl << np.uint64(2)) & np.uint64(0x3FFFC)) | np.uint64(4 * BIAS)
+    return b, tl >> np.uint64(16), u64(th & 0xFFFF), th >> 16
+
+
+def limbs_of(At):
+    """The same limbs taken straight from Ã (|Ã| < 2^62)."""
+    At = np.asarray(At, dtype=np.int64)
+    tl = u64(At & 0xFFFFFFFF)
+    th = At >> 32
+    b = ((tl & np.uint64(0xFFFF)) << np.uint64(2)) | np.uint64(4 * BIAS)
+    return b, tl >> np.uint64(16), u64(th & 0xFFFF), th >> 16
+
+
+def value_of(b, u1, u2, u3):
+    u0 = (b >> np.uint64(2)).astype(np.int64) - BIAS
+    return u0 + (u1.astype(np.int64) << 16) + (u2.astype(np.int64) << 32) + (u3 << 48)
+
+
+def limb_sum(b, u1, u2, u3, m, extra=0):
+    """Y = b + 4·extra + Σ u_j·4(2^16j mod m), wrapped to 32 bits, and the
+    same sum without wrapping."""
+    w = [4 * (pow(2, 16 * j, m)) for j in (1, 2, 3)]
+    exact = b.astype(np.int64) + 4 * extra + u1.astype(np.int64) * w[0] + u2.astype(np.int64) * w[1] + u3 * w[2]
+    Y = (b + np.uint64(4 * extra) + u1 * np.uint64(w[0]) + u2 * np.uint64(w[1])
+         + u64(u3 & 0xFFFFFFFF) * np.uint64(w[2])) & M32
+    return Y, exact
+
+
+def mulhi(a, b):
+    return (u64(a) * u64(b)) >> np.uint64(32)
+
+
+def residue_samples(rng, n=200_000):
+    lim = (1 << 62) - 1
+    At = rng.integers(-lim, lim, size=n, dtype=np.int64)
+    small = rng.integers(-(1 << 20), 1 << 20, size=n // 4, dtype=np.int64)
+    edges = np.array([0, 1, -1, lim, -lim, 1 << 32, -(1 << 32), (1 << 48) - 1, -(1 << 48),
+                      (1 << 16) - 1, -(1 << 16)], dtype=np.int64)
+    return np.concatenate([At, small, edges])
+
+
+def test_tz_quantiser_limbs():
+    """Normal, subnormal and zero entries at scales that keep |Ã| < 2^62, at
+    d = 1083 and at the zeroing scale -4096."""
+    rng = np.random.default_rng(5)
+    n = 200_000
+    sig = rng.uniform(0.5, 1.0, size=n) * rng.choice([-1.0, 1.0], size=n)
+    e = rng.integers(-1074, 1024, size=n)
+    x = np.ldexp(sig, e)
+    x = np.concatenate([x, np.ldexp(rng.uniform(-1, 1, size=n // 10), -1074 + rng.integers(0, 52, size=n // 10)),
+                        np.array([0.0, -0.0, 5e-324, -5e-324, np.finfo(float).max, -np.finfo(float).tiny])])
+    ex = np.frexp(x)[1]                       # |x| < 2^ex
+    dmax = np.minimum(TZ_FAST_MAX_D, 62 - ex)  # trunc(|x|·2^d) < 2^62
+    d = np.maximum(dmax - rng.integers(0, 120, size=x.size), -1100)
+    d = np.where(rng.random(x.size) < 0.02, -4096, d)
+    d = np.where(x == 0, rng.integers(-1100, TZ_FAST_MAX_D + 1, size=x.size), d)
+    got = value_of(*quantise_tz_limbs(x, d))
+    want = orc.quantise(x[:, None], d)[:, 0]
+    assert np.array_equal(got, want)
+
+
+def test_limb_split_round_trip():
+    rng = np.random.default_rng(6)
+    At = residue_samples(rng)
+    assert np.array_equal(value_of(*limbs_of(At)), At)
+
+
+@pytest.mark.parametrize("m", [m for m in orc.moduli(16) if not orc.square_base(m)])
+def test_nonsquare_table_index(m):
+    """Y - 4qm lies in [-4m, 4m), and entry m + (Y - 4qm)/4 of the rotated
+    table (entry i: the residue (i - 2^25) mod m) is Ã mod m."""
+    rng = np.random.default_rng(m)
+    At = residue_samples(rng)
+    b, u1, u2, u3 = limbs_of(At)
+    Y, exact = limb_sum(b, u1, u2, u3, m)
+    assert np.all((exact > 4 * (1 << 24)) & (exact < 4 * (1 << 28)))   # 2^24 < y < 2^28
+    assert np.array_equal(Y.astype(np.int64), exact)
+    magic = -(-(1 << 30) // m)
+    q = mulhi(Y, magic).astype(np.int64)
+    off = exact - q * 4 * m
+    assert np.all((off >= -4 * m) & (off < 4 * m) & (off % 4 == 0))
+    entry = m + off // 4
+    assert np.array_equal(np.mod(entry - BIAS, m), np.mod(At, m))
+
+
+@pytest.mark.parametrize("m", [m for m in orc.moduli(16) if orc.square_base(m)])
+def test_square_digits(m):
+    """The computed balanced base-s digits equal the oracle's digits of the
+    centred residue."""
+    s = orc.square_base(m)
+    H = m // 2
+    E = (H - BIAS) % m
+    h0 = s // 2
+    h1 = -(-(H - h0) // s)
+    shift = h0 + s * h1 - H
+    assert shift >= 0
+    rng = np.random.default_rng(m)
+    At = residue_samples(rng)
+    b, u1, u2, u3 = limbs_of(At)
+    Y, exact = limb_sum(b, u1, u2, u3, m, extra=E)
+    assert np.all((exact > 4 * (1 << 24)) & (exact < 4 * (1 << 28)))   # 2^24 < y < 2^28
+    assert np.array_equal(Y.astype(np.int64), exact)
+    q = mulhi(Y, -(-(1 << 30) // m)).astype(np.int64)
+    off = exact - q * 4 * m
+    off = np.where(off < 0, off + 4 * m, off)
+    u = (off >> 2) + shift
+    a1 = u >> 5 if s == 32 else mulhi(u, -(-(1 << 32) // s)).astype(np.int64)
+    a0 = u - a1 * s
+    d0, d1 = orc.square_digits(orc.centred(At, m), s)
+    assert np.array_equal(a0 - h0, d0) and np.array_equal(a1 - h1, d1)
