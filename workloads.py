@@ -34,7 +34,8 @@ class Workload:
 # The five dense shapes: a small case the oracle finishes in seconds, the
 # square 4096 case, the square 16384 ceiling case, a tall-K case stressing
 # K-chunking, and a k = 64 case with a wide dynamic range and 1% of A's rows
-# scaled by 2^±300 (native-FP64 fallback rows); and a batched-GEMV shape.
+# scaled by 2^±300 (native-FP64 fallback rows); a batched-GEMV shape; and a
+# small-C, long-k shape.
 WORKLOADS = {
     "dgemm_256": Workload("dgemm_256", 256, 256, 256, 0.5, 12, index=1),
     "dgemm_4096": Workload("dgemm_4096", 4096, 4096, 4096, 0.5, 12, index=2),
@@ -45,6 +46,9 @@ WORKLOADS = {
     # Batched GEMV (§3 "Strategy 1"): Y = A·X with a batch of 16 right-hand
     # sides, through the same kernels.
     "gemv_batch16": Workload("gemv_batch16", 16384, 16, 16384, 0.5, 12, index=6),
+    # A Gram-type block: a small C with a long k, which the residue GEMM
+    # splits along k.
+    "gram_256": Workload("gram_256", 256, 256, 65536, 0.5, 12, index=7),
 }
 
 
