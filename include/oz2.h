@@ -295,7 +295,9 @@ int oz2_deconstruct(int64_t m, int64_t n, int64_t k, int num_moduli,
  * element i·n·ldr; rows m..ldr-1 are not written).  Three FP8 tcgen05 MMAs
  * per modulus into two FP32 accumulators with exact accumulation (Eq.
  * accum-exact), reduced mod m_i every K-slab (32768 for square moduli, 4096
- * for nonsquare ones).  ldr < m → OZ2_ERR_INVALID_ARG. */
+ * for nonsquare ones).  This entry has no scratch, so it never splits k
+ * (oz2_dgemm_ex does for a small C with a long k; the results are the same).
+ * ldr < m → OZ2_ERR_INVALID_ARG. */
 int oz2_residue_gemm(int64_t m, int64_t n, int64_t k, int num_moduli,
                      const uint8_t* d_planes_a, const uint8_t* d_planes_b,
                      int16_t* d_residues, int64_t ldr, void* stream);
