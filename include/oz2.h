@@ -128,9 +128,11 @@ int oz2_dgemm_host(int64_t m, int64_t n, int64_t k,
  * a fixed 32 MiB array in the library's own device memory (held on every GPU
  * that loads the library until the process exits); problems whose
  * oz2_workspace_size exceeds 32 MiB (about 512³ at num_moduli = 16) return
- * OZ2_ERR_UNSUPPORTED.  It calls no allocation routine.  The first call on
- * each device looks up the array's device address and uploads the library's
- * digit-plane table; make that first call before any stream capture.  All
+ * OZ2_ERR_UNSUPPORTED.  It calls no allocation routine and creates no memory
+ * pool (the library's stream-ordered pool is made only by the entry points
+ * that allocate).  The first call on each device looks up the array's device
+ * address and uploads the library's digit-plane table with synchronous
+ * copies; make that first call before any stream capture.  All
  * calls share the one array: calls whose work overlaps on the GPU (different
  * streams, or concurrent host threads) race and must be serialised by the
  * caller.  Each call clears what it needs before using it. */
@@ -237,6 +239,18 @@ int oz2_get_stats(oz2_stats* out);
  * returns OZ2_ERR_TIMEOUT and clears the word.  OZ2_ERR_INVALID_ARG for a
  * limit out of range. */
 int oz2_selftest_timeout(long long limit_cycles, void* stream);
+
+/* Measurement probe for the FP8 tensor-pipe peak (the dense FP8 rate of the
+ * paper's hardware table, here measured rather than quoted).  Every CTA pair
+ * that can be resident issues `iters` (1 to 2^40) MMAs of the residue GEMM's
+ * own form, tcgen05.mma.cta_group::2.kind::f8f6f4 with M = N = 256, K = 32,
+ * on zero-filled operands in shared memory into one TMEM accumulator: no
+ * loads, no epilogue, no output.  The caller times the launch on `stream`;
+ * the work is (*cta_pairs)·iters·2·256·256·32 FP8 flops.  Writes the number
+ * of CTA pairs to *cta_pairs (if not null).  OZ2_ERR_INVALID_ARG for iters
+ * out of range; a wait that expires is reported by oz2_check_device_status
+ * as OZ2_ERR_TIMEOUT. */
+int oz2_probe_mma_rate(int64_t iters, int* cta_pairs, void* stream);
 
 /* oz2_dgemm, oz2_dgemm_host and oz2_fallback take their workspace and
  * staging buffers from a stream-ordered memory pool that the library owns on

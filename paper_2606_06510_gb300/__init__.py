@@ -69,6 +69,7 @@ _SIGS = {
     "oz2_trim_memory": (_I, []),
     "oz2_selftest_timeout": (_I, [ctypes.c_longlong, _P]),
     "oz2_check_device_status": (_I, []),
+    "oz2_probe_mma_rate": (_I, [_I64, _P, _P]),
     "oz2_status_string": (ctypes.c_char_p, [_I]),
     "oz2_scan": (_I, [_I64, _I64, _I64, _P, _I64, _P, _I64, _U, _P, _P, _P, _P, _P]),
     "oz2_scale": (_I, [_I64, _I64, _I64, _I, _P, _I64, _P, _I64, _P, _P, _P, _P, _I, _I, _P, _P, _P, _P, _P, _P]),
@@ -233,6 +234,15 @@ def oz2_get_stats() -> dict:
     out = {name: getattr(s, name) for name, _ in s._fields_ if name != "stage_ms"}
     out["stage_ms"] = dict(zip(STAGES, list(s.stage_ms)))
     return out
+
+
+def oz2_probe_mma_rate(iters: int, stream=None) -> int:
+    """Launch the tensor-pipe rate probe (iters MMAs of 256x256x32 FP8 per
+    CTA pair) on the stream; returns the number of CTA pairs it runs on."""
+    pairs = ctypes.c_int(0)
+    _check(lib().oz2_probe_mma_rate(iters, ctypes.cast(ctypes.pointer(pairs), ctypes.c_void_p), _stream(stream)),
+           "oz2_probe_mma_rate")
+    return pairs.value
 
 
 def oz2_check_device_status() -> int:

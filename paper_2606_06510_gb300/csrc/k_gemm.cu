@@ -490,6 +490,63 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
 }
 
 // ---------------------------------------------------------------------------
+// Tensor-pipe rate probe.  Every CTA pair issues `iters` MMAs of the residue
+// GEMM's own form (cta_group::2, kind::f8f6f4, M = N = 256, K = 32) on one
+// zero-filled operand tile pair in shared memory, into one accumulator, with
+// no loads and no epilogue.  Timed by the caller, it gives the dense FP8 rate
+// of the tensor pipes at the clock they run at: the ceiling for the residue
+// GEMM, which issues the same instruction.  The shared-memory request keeps
+// one CTA per SM, as in the GEMM.
+// ---------------------------------------------------------------------------
+constexpr int kProbeThreads = 64;
+constexpr size_t kProbeSmem = 1024 + 2 * kTileBytes + 64 + 128 * 1024;
+
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kProbeThreads, 1)
+    mma_rate_kernel(int64_t iters, Oz2Device* dev) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + 2 * kTileBytes);
+  __shared__ uint32_t tmem_base_s;
+  const int warp = threadIdx.x >> 5;
+  const bool leader = cluster_ctarank() == 0;
+  for (int i = threadIdx.x; i < 2 * kTileBytes / 16; i += kProbeThreads)
+    reinterpret_cast<uint4*>(smem)[i] = make_uint4(0u, 0u, 0u, 0u);
+  fence_proxy_async_smem();  // the tensor core reads what the threads wrote
+  if (threadIdx.x == 0) {
+    mbar_init(smem_u32(bar), 1);
+    fence_barrier_init();
+  }
+  if (warp == 1) {
+    tmem_alloc_pair(smem_u32(&tmem_base_s), kAccCols);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  cluster_sync_all();
+  tc_fence_after();
+  const uint32_t tmem = tmem_base_s;
+  if (leader && threadIdx.x == 32) {
+    constexpr uint32_t idesc = idesc_f8_f32(kTileM, kTileN);
+    const uint64_t a = smem_desc_sw128(smem_u32(smem)), b = a + (kTileBytes >> 4);
+    for (int64_t it = 0; it < iters; ++it) {
+      const uint32_t kk = static_cast<uint32_t>(it & 3);
+      mma_f8_pair(tmem, a + 2 * kk, b + 2 * kk, idesc, it ? 1u : 0u);
+    }
+    mma_commit_pair(smem_u32(bar));
+    if (!mbar_wait_bounded(smem_u32(bar), 0, kWaitLimit)) {
+      dev->status = kStatusTimeout;
+      dev->timeout_site = 4;
+    }
+  }
+  __syncwarp();
+  tc_fence_before();
+  cluster_sync_all();  // the pair's MMAs read both CTAs' shared memory
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc_pair(tmem, kAccCols);
+}
+
+cudaError_t launch_mma_rate(int64_t iters, Oz2Device* dev, int* pairs_out, cudaStream_t st);
+
+// ---------------------------------------------------------------------------
 // Plain CUDA-core kernel with the same semantics (diagnostic reference for
 // the tensor-core path; accumulates the same integer plane products in FP32
 // in sequential k order, so exactness follows from the same bound).
@@ -816,6 +873,34 @@ cudaError_t launch_plane_gemm(int64_t m, int64_t n, int64_t k_pad, const Oz2Modu
     count_launch();
     fold_parts_kernel<<<g, kFoldThreads, 0, st>>>(partials, residues, m, n, ldr, static_cast<int>(um.kparts), mods);
   }
+  return cudaGetLastError();
+}
+
+// The rate probe on as many CTA pairs as can be resident at once.
+cudaError_t launch_mma_rate(int64_t iters, Oz2Device* dev, int* pairs_out, cudaStream_t st) {
+  cudaError_t err =
+      cudaFuncSetAttribute(mma_rate_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kProbeSmem));
+  if (err != cudaSuccess) return err;
+  int64_t pairs = num_sms() / 2;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(2 * pairs));
+  cfg.blockDim = dim3(kProbeThreads);
+  cfg.dynamicSmemBytes = kProbeSmem;
+  cudaLaunchAttribute attr;
+  attr.id = cudaLaunchAttributeClusterDimension;
+  attr.val.clusterDim.x = 2;
+  attr.val.clusterDim.y = 1;
+  attr.val.clusterDim.z = 1;
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  int clusters = 0;
+  if (cudaOccupancyMaxActiveClusters(&clusters, mma_rate_kernel, &cfg) == cudaSuccess && clusters > 0)
+    pairs = std::min<int64_t>(pairs, clusters);
+  else
+    cudaGetLastError();
+  if (pairs_out) *pairs_out = static_cast<int>(pairs);
+  count_launch();
+  mma_rate_kernel<<<static_cast<unsigned>(2 * pairs), kProbeThreads, kProbeSmem, st>>>(iters, dev);
   return cudaGetLastError();
 }
 

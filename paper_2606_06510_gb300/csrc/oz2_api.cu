@@ -213,8 +213,10 @@ struct DeviceState {
   Oz2Device* status = nullptr;
   // Stream-ordered pool for the workspaces and staging buffers the library
   // allocates itself; it keeps freed blocks for reuse (release threshold:
-  // unlimited) until oz2_trim_memory.
+  // unlimited) until oz2_trim_memory.  Created by the first call that
+  // allocates, so entry points that allocate nothing never create it.
   cudaMemPool_t pool = nullptr;
+  bool pool_tried = false;
   // oz2_dgemm_host: a stream for copying finished column blocks of C back,
   // one event per block and one for the last copy, created on first use; the
   // mutex serialises host-buffer calls on this device, which share them.
@@ -290,28 +292,37 @@ static int device_state(DeviceState** out) {
       return OZ2_ERR_CUDA;
     s.table_a = tables;
     s.table_b = tables + kTableMax;
-    cudaMemPoolProps props;
-    std::memset(&props, 0, sizeof(props));
-    props.allocType = cudaMemAllocationTypePinned;
-    props.location.type = cudaMemLocationTypeDevice;
-    props.location.id = dev;
-    if (cudaMemPoolCreate(&s.pool, &props) == cudaSuccess) {
-      cuuint64_t keep = ~cuuint64_t(0);
-      cudaMemPoolSetAttribute(s.pool, cudaMemPoolAttrReleaseThreshold, &keep);
-    } else {
-      cudaGetLastError();
-      s.pool = nullptr;  // the device's default pool serves instead
-    }
     s.ready = true;
   }
   *out = &s;
   return OZ2_OK;
 }
 
-// Stream-ordered allocation from the library's pool on the current device.
+// Stream-ordered allocation from the library's pool on the current device
+// (the pool is created here, on the device's first allocation).
 static cudaError_t pool_alloc(void** p, size_t bytes, cudaStream_t s) {
   DeviceState* ds = nullptr;
   if (device_state(&ds) != OZ2_OK) return cudaErrorInitializationError;
+  {
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (!ds->pool_tried) {
+      ds->pool_tried = true;
+      int dev = 0;
+      cudaGetDevice(&dev);
+      cudaMemPoolProps props;
+      std::memset(&props, 0, sizeof(props));
+      props.allocType = cudaMemAllocationTypePinned;
+      props.location.type = cudaMemLocationTypeDevice;
+      props.location.id = dev;
+      if (cudaMemPoolCreate(&ds->pool, &props) == cudaSuccess) {
+        cuuint64_t keep = ~cuuint64_t(0);
+        cudaMemPoolSetAttribute(ds->pool, cudaMemPoolAttrReleaseThreshold, &keep);
+      } else {
+        cudaGetLastError();
+        ds->pool = nullptr;  // the device's default pool serves instead
+      }
+    }
+  }
   return ds->pool ? cudaMallocFromPoolAsync(p, bytes, ds->pool, s) : cudaMallocAsync(p, bytes, s);
 }
 
@@ -808,6 +819,14 @@ int oz2_selftest_timeout(long long limit_cycles, void* stream) {
   count_launch();
   timeout_probe_kernel<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(ds->status, limit_cycles);
   return to_status(cudaGetLastError());
+}
+
+int oz2_probe_mma_rate(int64_t iters, int* cta_pairs, void* stream) {
+  if (iters < 1 || iters > (int64_t{1} << 40)) return OZ2_ERR_INVALID_ARG;
+  DeviceState* ds = nullptr;
+  const int st = device_state(&ds);
+  if (st) return st;
+  return to_status(launch_mma_rate(iters, ds->status, cta_pairs, static_cast<cudaStream_t>(stream)));
 }
 
 int oz2_check_device_status(void) {

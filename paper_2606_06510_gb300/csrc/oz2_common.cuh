@@ -438,6 +438,8 @@ cudaError_t launch_fallback_lists(int64_t m, int64_t n, int64_t k, const double*
                                   const double* B, int64_t ldb, const uint8_t* row_flag,
                                   const uint8_t* col_flag, int* scratch, double* C, int64_t ldc,
                                   cudaStream_t st, bool zero_counts);
+// The tensor-pipe rate probe (k_gemm.cu); reports the CTA pairs it runs on.
+cudaError_t launch_mma_rate(int64_t iters, Oz2Device* dev, int* pairs_out, cudaStream_t st);
 cudaError_t launch_native(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda,
                           const double* B, int64_t ldb, double* C, int64_t ldc, cudaStream_t st);
 }  // namespace oz2

@@ -17,7 +17,7 @@ def oz():
 
 def test_every_header_symbol_is_exported(oz):
     names = header_functions()
-    assert len(names) == 21
+    assert len(names) == 22
     raw = ctypes.CDLL(oz.LIB_PATH)
     missing = [n for n in names if not hasattr(raw, n)]
     assert not missing

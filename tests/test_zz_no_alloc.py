@@ -14,6 +14,7 @@ import pytest
 
 import workloads as wl
 from helpers import ensure_built, to_dev
+from oracle import ozaki2 as orc
 
 pytestmark = pytest.mark.gpu
 
@@ -69,3 +70,42 @@ def test_rejects_problems_beyond_the_scratch(env):
     assert oz.oz2_workspace_size(m, n, k, 12) > LIMIT
     rc = f(m, n, k, None, m, None, k, None, m, 12, None)   # rejected before any device work
     assert rc == -6          # OZ2_ERR_UNSUPPORTED
+
+
+def test_matches_the_oracle(env):
+    """One call checked directly against the oracle (not only against
+    oz2_dgemm), bit for bit, with a fallback row and a zero column."""
+    m, n, k, r = 200, 136, 300, 12
+    A = np.array(wl.random_matrix(m, k, 1.0, 4242), order="F")
+    B = np.array(wl.random_matrix(k, n, 1.0, 4243), order="F")
+    A[7, :] *= 2.0 ** 300
+    B[:, 40] = 0.0
+    got = call_noalloc(env, to_dev(A), to_dev(B), r)
+    want = orc.oz2_dgemm(A, B, r).C
+    same = (got == want) | (np.isnan(got) & np.isnan(want))
+    assert same.all(), f"{(~same).sum()} entries differ from the oracle"
+
+
+@pytest.mark.parametrize("shape,r,parts", [((64, 64, 3000), 12, 4), ((128, 64, 2500), 14, 2)])
+def test_split_k_in_the_scratch_then_an_unsplit_call(env, shape, r, parts):
+    """A small C with a long k: the residue GEMM splits k and keeps the
+    parts' residues in the scratch array's magnitude-plane region.  The
+    split call (one launch more than an unsplit one: the fold) must match
+    oz2_dgemm bit for bit, and an unsplit call right after it must too."""
+    oz, _, _ = env
+    m, n, k = shape
+    assert oz.oz2_workspace_size(m, n, k, r) <= LIMIT
+    assert oz.oz2_plan(m, n, k, r, 76)["kparts"] == parts
+    A = to_dev(wl.random_matrix(m, k, 1.0, 5151 + r))
+    B = to_dev(wl.random_matrix(k, n, 1.0, 5252 + r))
+    oz.oz2_get_stats()                      # resets the launch counter
+    got = call_noalloc(env, A, B, r)
+    assert oz.oz2_get_stats()["kernel_launches"] == 13
+    want = oz.oz2_dgemm(A, B, num_moduli=r).cpu().numpy()
+    assert np.array_equal(got, want)
+    A2 = to_dev(wl.random_matrix(96, 300, 0.5, 5353 + r))
+    B2 = to_dev(wl.random_matrix(300, 80, 0.5, 5454 + r))
+    oz.oz2_get_stats()
+    got2 = call_noalloc(env, A2, B2, r)
+    assert oz.oz2_get_stats()["kernel_launches"] == 12
+    assert np.array_equal(got2, oz.oz2_dgemm(A2, B2, num_moduli=r).cpu().numpy())
