@@ -3,10 +3,13 @@
 // and one correctly rounded (round-to-nearest-even) conversion of
 // X·2^-(d_i+e_j) to FP64, including the subnormal range.
 //
-// X is computed by the direct CRT sum in fixed point (multiply-adds only);
-// Garner's algorithm, the paper's method, takes over in the rare case where
-// the fixed-point quotient is ambiguous, so every output equals the Garner
-// result exactly.
+// X is computed by the direct CRT sum in fixed point (multiply-adds only).
+// For r = 11 and 12 one 96-bit sum estimates X to about 2^28 and decides the
+// rounding whenever no midpoint between doubles lies that close; the other
+// outputs, and every output at other r, take an exact two-word or five-limb
+// direct CRT, and Garner's algorithm, the paper's method, takes over in the
+// rare case where that sum's quotient is ambiguous.  Every output equals
+// the Garner result exactly.
 //
 // Residues arrive column-major (r matrices of m×n, ld = ldr ≥ m) from the
 // residue GEMM and C is column-major, so a thread takes two consecutive
@@ -14,9 +17,9 @@
 // modulus) and one 16-byte store of its two results (a warp writes 512
 // contiguous bytes), with no transposition.  Each thread walks a strided
 // set of columns and loads the next column's residues while it computes the
-// current one.  An output that needs Garner's algorithm is marked with a
-// NaN sentinel and recomputed after the loop, which keeps Garner's register
-// footprint out of the loop.
+// current one.  An output that the fast path leaves is marked with a NaN
+// sentinel and recomputed after the loop, which keeps the exact paths'
+// register footprint out of the loop.
 #include "oz2_common.cuh"
 
 namespace oz2 {
@@ -307,15 +310,107 @@ __device__ __forceinline__ bool crt_value_w64(const int (&c)[R], int E, const Oz
   return true;
 }
 
+// Fast path for r = 11, 12 (2^102 < M < 2^112): one 96-bit fixed-point sum.
+// With F_k = round(2^96·y_k/m_k), Y = Σ c_k F_k mod 2^96 read as a signed
+// word is 2^96·X/M + D with |D| ≤ Σ|c_k|/2, as long as that stays inside
+// [-2^95, 2^95) (|Y| < 2^95 - 2^64 shows there was no wrap).  Then
+// P = ⌊|Y|·M/2^96⌋, from the partial products of |Y|'s and M's 32-bit words
+// at or above 2^64, is within err (a host-computed bound, about 2^27.7 for
+// centred residues) of |X|, and X has Y's sign.  With P of b bits, T = P >> s
+// (s = b - 64) holds P's leading 64 bits and rounds to 53 at its bit 11, so
+// the midpoint between two doubles sits at bit s + 10 of P.  W, bits
+// s - 21 .. s + 10 of P, puts that midpoint at bit 31; when W is more than
+// e_W = ⌊err/2^(s-21)⌋ + 2 from 2^31, no midpoint lies between |X| and P,
+// and the hardware conversion of T, with bit 0 set when W is above 2^31
+// (T's own bits may sit exactly on the midpoint), rounds as |X| would
+// (e_W < 2^29 keeps the midpoints of the binade below out of reach too).
+// Returns false (the caller takes an exact path) when |Y| is too close to
+// 2^95, when P < 2^85, when the test fails, or when the result would not be
+// a normal double.
+template <int R>
+__device__ __forceinline__ bool crt_value_y96(const int (&c)[R], int E, const Oz2Moduli& mods,
+                                              unsigned long long err, double& out) {
+  long long a0 = 0, a1 = 0;
+  uint32_t a2 = 0;
+#pragma unroll
+  for (int k = 0; k < R; ++k) {
+    a0 += static_cast<long long>(c[k]) * mods.crt_y0[k];
+    a1 += static_cast<long long>(c[k]) * mods.crt_y1[k];
+    a2 += static_cast<uint32_t>(c[k]) * mods.crt_y2[k];
+  }
+  // Y = a0 + a1·2^32 + a2·2^64 (mod 2^96) as words w2:w1:w0.
+  const long long s1 = (a0 >> 32) + a1;
+  const uint32_t w0 = static_cast<uint32_t>(a0), w1 = static_cast<uint32_t>(s1);
+  const uint32_t w2 = static_cast<uint32_t>(static_cast<u64>(s1) >> 32) + a2;
+  const uint32_t sg = static_cast<uint32_t>(static_cast<int>(w2) >> 31);  // 0 or all ones
+  // |Y| = (Y ^ sg) - sg
+  const u64 lo = ((static_cast<u64>(w1 ^ sg) << 32) | (w0 ^ sg)) - static_cast<u64>(static_cast<long long>(static_cast<int>(sg)));
+  const uint32_t y2 = (w2 ^ sg) + ((sg != 0u && lo == 0) ? 1u : 0u);
+  if (y2 >= 0x7FFFFFFFu) return false;
+  const uint32_t y0 = static_cast<uint32_t>(lo), y1 = static_cast<uint32_t>(lo >> 32);
+  const uint32_t m0 = mods.crt_m32[0], m1 = mods.crt_m32[1], m2 = mods.crt_m32[2], m3 = mods.crt_m32[3];
+  // P = Σ_{i+j≥2} y_i m_j 2^(32(i+j) - 96), the i + j = 2 products by their
+  // high words: col3 (at 2^0, three products), col4 (at 2^32, two), col5
+  // (at 2^64, one; m3 < 2^16).
+  const u64 c2 = static_cast<u64>(__umulhi(y0, m2)) + __umulhi(y1, m1) + __umulhi(y2, m0);
+  const u64 t0 = static_cast<u64>(y0) * m3 + c2;
+  const u64 t1 = static_cast<u64>(y1) * m2;
+  const u64 t2 = static_cast<u64>(y2) * m1;
+  const u64 col4 = static_cast<u64>(y1) * m3 + static_cast<u64>(y2) * m2;
+  const u64 s01 = t0 + t1;
+  const u64 s012 = s01 + t2;
+  const u64 pl = s012 + (col4 << 32);
+  const u64 ph = static_cast<u64>(y2) * m3 + (col4 >> 32) + (s01 < t0 ? 1u : 0u) + (s012 < s01 ? 1u : 0u) +
+                 (pl < s012 ? 1u : 0u);
+  const int lz = __clzll(static_cast<long long>(ph));  // P has 128 - lz bits
+  if (lz > 43) return false;                            // P < 2^85 (or ph = 0)
+  const int sh = 64 - lz;                               // T = P >> sh, sh in [21, 48]
+  const int u = sh - 21;
+  const u64 ew = (err >> u) + 2;
+  const uint32_t W = static_cast<uint32_t>(pl >> u);
+  if (ew >= (1ull << 29) || static_cast<uint32_t>(W - 0x80000000u + static_cast<uint32_t>(ew)) <=
+                                2u * static_cast<uint32_t>(ew))
+    return false;
+  // W ≥ 2^31 (never equal here) puts P above the midpoint of T's rounding
+  // cell: bit 0 then makes a T whose low 11 bits are exactly 1024 round up.
+  const u64 top = (ph << lz) | (pl >> sh) | (W >> 31);
+  const int e2 = 127 - lz + E;                          // exponent of P's leading bit, scaled
+  if (e2 < -1022 || e2 > 1022) return false;
+  const long long bits = __double_as_longlong(__ull2double_rn(top)) + (static_cast<long long>(E + sh) << 52);
+  out = __longlong_as_double(bits | (sg ? (1ll << 63) : 0ll));
+  return true;
+}
+
 constexpr int kCrtThreads = 256;
 constexpr long long kCrtSentinel = 0x7FF4DEAD0BADF00Dll;  // a NaN the reconstruction never produces
 
+// The fast path by moduli count: the 96-bit estimate for r = 11, 12 (M of
+// 103 and 112 bits: |X| is then above 2^85 except in rare outputs); the
+// exact two-word CRT for r ≤ 10, where X has at most 94 bits and an
+// estimate within ±err decides fewer roundings; the five-limb CRT for
+// r ≥ 13.
 template <int R>
-__device__ __forceinline__ bool crt_fast(const int (&c)[R], int E, const Oz2Moduli& mods, double& out) {
-  if constexpr (R <= 12)
+__device__ __forceinline__ bool crt_fast(const int (&c)[R], int E, const Oz2Moduli& mods, unsigned long long err,
+                                         double& out) {
+  if constexpr (R >= 11 && R <= 12)
+    return crt_value_y96<R>(c, E, mods, err, out);
+  else if constexpr (R <= 10)
     return crt_value_w64<R>(c, E, mods, out);
   else
     return crt_value_fast<R>(c, E, mods, out);
+}
+
+// The exact paths, for outputs the fast path leaves: the two-word direct CRT
+// (r ≤ 12) or the five-limb one, then Garner's algorithm.
+template <int R>
+__device__ __noinline__ double crt_exact(const int (&c)[R], int E, const Oz2Moduli& mods) {
+  double v;
+  if constexpr (R <= 12) {
+    if (crt_value_w64<R>(c, E, mods, v)) return v;
+  } else {
+    if (crt_value_fast<R>(c, E, mods, v)) return v;
+  }
+  return crt_value<R>(c, E, mods);
 }
 
 // Resident blocks per SM the register budget is sized for: the two-word
@@ -333,9 +428,10 @@ constexpr int crt_min_blocks() {
 // loads and 16-byte stores possible; otherwise element-wise accesses.
 // Returns how many outputs were left to Garner's algorithm.
 template <int R, bool FAST>
-__device__ __forceinline__ int crt_columns(int64_t n, int64_t row, bool pair, int d0, int d1,
-                                           const Oz2Moduli& mods, const int16_t* __restrict__ res, int64_t ldr,
-                                           const int* __restrict__ e, double* cbase, int64_t ldc) {
+__device__ __forceinline__ uint32_t crt_columns(int64_t n, int64_t row, bool pair, int d0, int d1,
+                                                const Oz2Moduli& mods, unsigned long long err,
+                                                const int16_t* __restrict__ res, int64_t ldr,
+                                                const int* __restrict__ e, double* cbase, int64_t ldc) {
   const int64_t step = gridDim.y;
   const int64_t off_step = step * ldr;
   // Residue matrix k starts at res + k·mstride (the same for every thread,
@@ -356,7 +452,10 @@ __device__ __forceinline__ int crt_columns(int64_t n, int64_t row, bool pair, in
         w[k] = static_cast<uint16_t>(base[k][off]) | (pair ? static_cast<uint32_t>(base[k][off + 1]) << 16 : 0u);
     }
   };
-  int pending = 0;
+  // Bit j: the j-th column of this thread has an output left to the exact
+  // path (bit 31: one of the 32nd or later columns has).
+  uint32_t pending = 0;
+  int iter = 0;
   auto column = [&](const uint32_t (&w)[R], int ec, int64_t col) {
     double v[2];
 #pragma unroll
@@ -366,12 +465,13 @@ __device__ __forceinline__ int crt_columns(int64_t n, int64_t row, bool pair, in
       for (int k = 0; k < R; ++k)
         c[k] = u ? (static_cast<int>(w[k]) >> 16) : static_cast<int>(static_cast<int16_t>(w[k] & 0xFFFFu));
       double val;
-      if (!crt_fast<R>(c, -((u ? d1 : d0) + ec), mods, val)) {
+      if (!crt_fast<R>(c, -((u ? d1 : d0) + ec), mods, err, val)) {
         val = __longlong_as_double(kCrtSentinel);
-        ++pending;
+        pending |= 1u << (iter < 31 ? iter : 31);
       }
       v[u] = val;
     }
+    ++iter;
     double* out = cbase + col * ldc;
     if (FAST) {
       *reinterpret_cast<double2*>(out) = make_double2(v[0], v[1]);
@@ -414,26 +514,34 @@ __device__ __forceinline__ int crt_columns(int64_t n, int64_t row, bool pair, in
 template <int R, bool FAST>
 __global__ void __launch_bounds__(kCrtThreads, crt_min_blocks<R, FAST>())
     crt_kernel(int64_t row0, int64_t rows, int64_t n, const __grid_constant__ Oz2Moduli mods,
-               const int16_t* __restrict__ res, int64_t ldr, const int* __restrict__ d, const int* __restrict__ e,
-               double* __restrict__ C, int64_t ldc) {
+               unsigned long long err, const int16_t* __restrict__ res, int64_t ldr, const int* __restrict__ d,
+               const int* __restrict__ e, double* __restrict__ C, int64_t ldc) {
   const int64_t rel = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) * 2;
   if (rel >= rows) return;
   const int64_t row = row0 + rel;
   const bool pair = rel + 1 < rows;
   const int d0 = d[row], d1 = pair ? d[row + 1] : 0;
   double* cbase = C + row;
-  const int pending = crt_columns<R, FAST>(n, row, pair, d0, d1, mods, res, ldr, e, cbase, ldc);
+  uint32_t pending = crt_columns<R, FAST>(n, row, pair, d0, d1, mods, err, res, ldr, e, cbase, ldc);
   if (pending == 0) return;
-  // Outputs the fast path left to Garner's algorithm (this thread's own).
+  // Outputs the fast path left to the exact paths (this thread's own): the
+  // columns its mask marks, and every column from the 32nd on if bit 31 is set.
   const int64_t step = gridDim.y;
-  for (int64_t col = blockIdx.y; col < n; col += step) {
-    for (int u = 0; u < (pair ? 2 : 1); ++u) {
-      double* q = cbase + col * ldc + u;
-      if (__double_as_longlong(*q) != kCrtSentinel) continue;
-      int c[R];
+  const int64_t tail = blockIdx.y + 31 * step;
+  while (pending) {
+    const int j = __ffs(pending) - 1;
+    pending &= pending - 1;
+    const int64_t c_lo = blockIdx.y + j * step;
+    const int64_t c_hi = j < 31 ? c_lo + 1 : n;
+    for (int64_t col = j < 31 ? c_lo : tail; col < c_hi && col < n; col += (j < 31 ? 1 : step)) {
+      for (int u = 0; u < (pair ? 2 : 1); ++u) {
+        double* q = cbase + col * ldc + u;
+        if (__double_as_longlong(*q) != kCrtSentinel) continue;
+        int c[R];
 #pragma unroll
-      for (int k = 0; k < R; ++k) c[k] = res[(k * n + col) * ldr + row + u];
-      *q = crt_value<R>(c, -((u ? d1 : d0) + __ldg(e + col)), mods);
+        for (int k = 0; k < R; ++k) c[k] = res[(k * n + col) * ldr + row + u];
+        *q = crt_exact<R>(c, -((u ? d1 : d0) + __ldg(e + col)), mods);
+      }
     }
   }
 }
@@ -442,8 +550,8 @@ __global__ void __launch_bounds__(kCrtThreads, crt_min_blocks<R, FAST>())
 // over the columns, about two waves of resident blocks in all.
 template <int R, bool FAST>
 static cudaError_t launch_crt_rows(cudaStream_t st, int64_t row0, int64_t rows, int64_t n, const Oz2Moduli& mods,
-                                   const int16_t* res, int64_t ldr, const int32_t* d, const int32_t* e, double* C,
-                                   int64_t ldc) {
+                                   unsigned long long err, const int16_t* res, int64_t ldr, const int32_t* d,
+                                   const int32_t* e, double* C, int64_t ldc) {
   int dev = 0, sms = 148;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
@@ -455,31 +563,34 @@ static cudaError_t launch_crt_rows(cudaStream_t st, int64_t row0, int64_t rows, 
   gy = gy > 65535 ? 65535 : gy;
   count_launch();
   crt_kernel<R, FAST><<<dim3(static_cast<unsigned>(gx), static_cast<unsigned>(gy)), kCrtThreads, 0, st>>>(
-      row0, rows, n, mods, res, ldr, d, e, C, ldc);
+      row0, rows, n, mods, err, res, ldr, d, e, C, ldc);
   return cudaGetLastError();
 }
 
 template <int R>
-static cudaError_t launch_crt_r(cudaStream_t st, int64_t m, int64_t n, const Oz2Moduli& mods, const int16_t* res,
-                                int64_t ldr, const int32_t* d, const int32_t* e, double* C, int64_t ldc) {
+static cudaError_t launch_crt_r(cudaStream_t st, int64_t m, int64_t n, const Oz2Moduli& mods,
+                                unsigned long long e96, const int16_t* res, int64_t ldr, const int32_t* d,
+                                const int32_t* e, double* C, int64_t ldc) {
   const bool vec = (ldr % 2 == 0) && (reinterpret_cast<uintptr_t>(res) % 4 == 0) && (ldc % 2 == 0) &&
                    (reinterpret_cast<uintptr_t>(C) % 16 == 0);
-  if (!vec) return launch_crt_rows<R, false>(st, 0, m, n, mods, res, ldr, d, e, C, ldc);
+  if (!vec) return launch_crt_rows<R, false>(st, 0, m, n, mods, e96, res, ldr, d, e, C, ldc);
   const int64_t even = m & ~int64_t{1};
   cudaError_t err = cudaSuccess;
-  if (even > 0) err = launch_crt_rows<R, true>(st, 0, even, n, mods, res, ldr, d, e, C, ldc);
-  if (err == cudaSuccess && even < m) err = launch_crt_rows<R, false>(st, even, 1, n, mods, res, ldr, d, e, C, ldc);
+  if (even > 0) err = launch_crt_rows<R, true>(st, 0, even, n, mods, e96, res, ldr, d, e, C, ldc);
+  if (err == cudaSuccess && even < m)
+    err = launch_crt_rows<R, false>(st, even, 1, n, mods, e96, res, ldr, d, e, C, ldc);
   return err;
 }
 
 cudaError_t launch_reconstruct(int64_t m, int64_t n, const Oz2Moduli& mods, const int16_t* residues,
                                int64_t ldr, const int32_t* d, const int32_t* e, double* C, int64_t ldc,
-                               cudaStream_t st) {
+                               bool centred, cudaStream_t st) {
   if (m == 0 || n == 0) return cudaSuccess;
+  const unsigned long long e96 = centred ? mods.crt_err_centred : mods.crt_err_any;
   switch (mods.r) {
 #define OZ2_CRT_CASE(R) \
   case R:               \
-    return launch_crt_r<R>(st, m, n, mods, residues, ldr, d, e, C, ldc);
+    return launch_crt_r<R>(st, m, n, mods, e96, residues, ldr, d, e, C, ldc);
     OZ2_CRT_CASE(1) OZ2_CRT_CASE(2) OZ2_CRT_CASE(3) OZ2_CRT_CASE(4) OZ2_CRT_CASE(5) OZ2_CRT_CASE(6)
     OZ2_CRT_CASE(7) OZ2_CRT_CASE(8) OZ2_CRT_CASE(9) OZ2_CRT_CASE(10) OZ2_CRT_CASE(11) OZ2_CRT_CASE(12)
     OZ2_CRT_CASE(13) OZ2_CRT_CASE(14) OZ2_CRT_CASE(15) OZ2_CRT_CASE(16)

@@ -188,6 +188,35 @@ static Oz2Moduli build_moduli(int r, int quant) {
   u64 M[3] = {1, 0, 0};
   for (int i = 0; i < r; ++i) mul3(M, static_cast<u64>(kModuliAll[i]));
   for (int i = 0; i < 3; ++i) c.M[i] = M[i];
+  // 96-bit constants (used for r ≤ 12, M < 2^112): F_k = round(2^96·y_k/m_k)
+  // split into signed low words, and the error bound of the estimate of |X|:
+  // |X| - ⌊|Y|·M/2^96⌋ (partial products below 2^64 dropped) is within
+  // (Σ_k cmax_k)·M/2^97 + 5 < (Σ cmax_k)·(⌊M/2^64⌋ + 1)/2^33 + 5, with cmax_k
+  // = ⌊m_k/2⌋ for centred residues and 2^15 for any int16 residue.
+  {
+    u64 sum_centred = 0;
+    for (int k = 0; k < r; ++k) {
+      const int mk = kModuliAll[k];
+      long long pm = 1;
+      for (int j = 0; j < r; ++j)
+        if (j != k) pm = (pm * kModuliAll[j]) % mk;
+      const int y = mod_inverse(pm, mk);
+      const unsigned __int128 F = ((static_cast<unsigned __int128>(y) << 96) + static_cast<unsigned>(mk / 2)) / mk;
+      int lo = 0, hi = 0;
+      split_signed_low(static_cast<u64>(F), &lo, &hi);
+      c.crt_y0[k] = lo;
+      const unsigned __int128 F1 = (F - static_cast<unsigned __int128>(static_cast<__int128>(lo))) >> 32;
+      split_signed_low(static_cast<u64>(F1), &lo, &hi);
+      c.crt_y1[k] = lo;
+      c.crt_y2[k] = static_cast<uint32_t>((F1 - static_cast<unsigned __int128>(static_cast<__int128>(lo))) >> 32);
+      sum_centred += static_cast<u64>(mk / 2);
+    }
+    for (int i = 0; i < 4; ++i) c.crt_m32[i] = static_cast<uint32_t>(M[i >> 1] >> (32 * (i & 1)));
+    const unsigned __int128 mh1 = static_cast<unsigned __int128>(M[1]) + 1;  // M < 2^128 here
+    const u64 sum_any = 32768ull * static_cast<u64>(r);
+    c.crt_err_centred = static_cast<u64>((sum_centred * mh1 + ((static_cast<unsigned __int128>(1) << 33) - 1)) >> 33) + 6;
+    c.crt_err_any = static_cast<u64>((sum_any * mh1 + ((static_cast<unsigned __int128>(1) << 33) - 1)) >> 33) + 6;
+  }
   split_signed_low(M[0], &c.crt_ml, &c.crt_mlh);
   // round(M/2^51), below 2^61 while M < 2^112 (r ≤ 12, the only use).
   split_signed_low(((M[0] >> 51) | (M[1] << 13)) + ((M[0] >> 50) & 1), &c.crt_m51l, &c.crt_m51h);
@@ -574,7 +603,8 @@ static int run_stages(int64_t m, int64_t n, int64_t k, const double* A, int64_t 
     err = launch_plane_gemm(m, cols, L.k_pad, mods, pa, pb0, simt ? 2 : 0, res, L.res_ld, nullptr, ds->status, s,
                             reinterpret_cast<int16_t*>(mag_a), L.planes_a - L.mag_a);
     mark(6);
-    if (err == cudaSuccess) err = launch_reconstruct(m, cols, mods, res, L.res_ld, d, e + c0, C + c0 * ldc, ldc, s);
+    if (err == cudaSuccess)
+      err = launch_reconstruct(m, cols, mods, res, L.res_ld, d, e + c0, C + c0 * ldc, ldc, true, s);
     mark(7);
     if (err == cudaSuccess)
       err = launch_fallback_lists(m, cols, k, A, lda, B + c0 * ldb, ldb, rf, cf + c0, misc, C + c0 * ldc, ldc, s,
@@ -936,7 +966,8 @@ int oz2_reconstruct(int64_t m, int64_t n, int num_moduli, const int16_t* residue
   if (num_moduli < 1 || num_moduli > kMaxModuli) return OZ2_ERR_UNSUPPORTED_R;
   if (m && n && (!residues || !d || !e || !C)) return OZ2_ERR_INVALID_ARG;
   const Oz2Moduli mods = build_moduli(num_moduli, OZ2_QUANT_TZ);
-  return to_status(launch_reconstruct(m, n, mods, residues, ldr, d, e, C, ldc, static_cast<cudaStream_t>(stream)));
+  return to_status(
+      launch_reconstruct(m, n, mods, residues, ldr, d, e, C, ldc, false, static_cast<cudaStream_t>(stream)));
 }
 
 int oz2_fallback(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, const double* B, int64_t ldb,

@@ -139,6 +139,13 @@ struct Oz2Moduli {
   int crt_g[kMaxModuli];
   int crt_ml, crt_mlh;
   int crt_m51l, crt_m51h;
+  // 96-bit direct CRT (r = 11, 12): F_k = round(2^96·y_k/m_k) = y2·2^64 + y1·2^32 + y0
+  // with y0 and y1 signed low words; M as four 32-bit words; and bounds on
+  // |X| - ⌊|Y|·M/2^96⌋ for centred residues and for any int16 residues.
+  int crt_y0[kMaxModuli], crt_y1[kMaxModuli];
+  uint32_t crt_y2[kMaxModuli];
+  uint32_t crt_m32[4];
+  unsigned long long crt_err_centred, crt_err_any;
   int table_entries;            // 2·Σ m_i over the nonsquare moduli (digit-plane table)
 };
 
@@ -431,9 +438,11 @@ cudaError_t launch_plane_gemm(int64_t m, int64_t n, int64_t k_pad, const Oz2Modu
                               const uint8_t* planes_a, const uint8_t* planes_b, int mode,
                               int16_t* residues, int64_t ldr, float* urow, Oz2Device* dev, cudaStream_t st,
                               int16_t* partials = nullptr, size_t partial_bytes = 0);
+// `centred`: every residue lies in [-⌊m_k/2⌋, m_k-1-⌊m_k/2⌋] (as the residue
+// GEMM writes them); otherwise any int16 representative.
 cudaError_t launch_reconstruct(int64_t m, int64_t n, const Oz2Moduli& mods,
                                const int16_t* residues, int64_t ldr, const int32_t* d,
-                               const int32_t* e, double* C, int64_t ldc, cudaStream_t st);
+                               const int32_t* e, double* C, int64_t ldc, bool centred, cudaStream_t st);
 cudaError_t launch_fallback_lists(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda,
                                   const double* B, int64_t ldb, const uint8_t* row_flag,
                                   const uint8_t* col_flag, int* scratch, double* C, int64_t ldc,

@@ -248,6 +248,42 @@ def test_reconstruct_near_the_range_boundary(oz):
                 assert C[i, j] == want and np.signbit(C[i, j]) == np.signbit(want), (r, i, j)
 
 
+def test_reconstruct_next_to_rounding_midpoints(oz):
+    """Integers X placed at and around the midpoints between doubles of
+    X·2^E, at several bit lengths, where the fixed-point fast path must
+    defer to an exact path unless its estimate decides the rounding."""
+    import random
+    import torch
+    for r in (9, 11, 12):
+        mods = orc.moduli(r)
+        M = orc.modulus_product(mods)
+        rng = random.Random(100 + r)
+        xs = []
+        for b in range(max(60, M.bit_length() - 40), M.bit_length() - 1, 3):
+            q = b - 53
+            for off in (0, 1, -1, 1 << 20, -(1 << 20), 1 << 30, -(1 << 30), 1 << 34, -(1 << 34), 1 << 36):
+                if off and abs(off) >= 1 << (q - 1):
+                    continue
+                x = (rng.randrange(1 << 52, 1 << 53) << q) + (1 << (q - 1)) + off
+                if x < M // 2:
+                    xs.append(x * rng.choice((1, -1)))
+        xs += [rng.randrange(-(M // 2), M // 2) for _ in range(40)]
+        m, n = len(xs), 2
+        R = np.zeros((r, m, n), dtype=np.int64)
+        for i, x in enumerate(xs):
+            for k, mk in enumerate(mods):
+                R[k, i, :] = int(orc.centred(x % mk, mk))
+        d = np.full(m, 3, dtype=np.int64)
+        e = np.array([-M.bit_length(), 60], dtype=np.int64)
+        res = torch.from_numpy(R.astype(np.int16)).cuda()
+        C = oz.oz2_reconstruct(res, torch.from_numpy(d.astype(np.int32)).cuda(),
+                               torch.from_numpy(e.astype(np.int32)).cuda(), m, n, r).cpu().numpy()
+        for i, x in enumerate(xs):
+            for j in range(n):
+                want = orc.unscale_one(x, -int(d[i]) - int(e[j]))
+                assert C[i, j] == want and np.signbit(C[i, j]) == np.signbit(want), (r, i, j)
+
+
 def test_reconstruct_other_representatives(oz):
     """Residues in (-m_i, m_i) that are not the centred ones give the same
     results as the centred ones (the reconstruction's input contract)."""
