@@ -63,6 +63,14 @@ typedef enum { OZ2_SCALE_R2 = 0, OZ2_SCALE_R1 = 1 } oz2_scale_mode;
 #define OZ2_FLAG_TIMING      0x2u   /* record per-stage CUDA events on the stream;
                                        harvested by oz2_get_stats (no host sync
                                        inside the call) */
+/* For num_moduli 11 or 12 and k ≤ 256: run the residue GEMM and the
+ * reconstruction fused in one kernel, each output's residues folded into
+ * its CRT sum on chip (Algorithm 1 Phase 3 in the GEMM epilogue), instead of
+ * two launches through the residue matrices.  It moves fewer DRAM bytes
+ * (no 2r bytes per output written and read back) but streams every plane of
+ * A through L2 once per 32 columns of C, and on one GB300 it measured slower
+ * than the two launches for every shape tried; see oz2_dgemm_ex. */
+#define OZ2_FLAG_FUSED       0x4u
 /* Diagnostic only: run the "+1" and residue plane GEMMs on CUDA cores with
  * the same integer plane products and epilogue arithmetic (slow; used by
  * the tests to separate tensor-core issues from the rest of the path). */
@@ -149,7 +157,11 @@ size_t oz2_workspace_size(int64_t m, int64_t n, int64_t k, int num_moduli);
  * (oz2_scale_mode), flags (OZ2_FLAG_*) and caller-provided device workspace of
  * ws_bytes ≥ oz2_workspace_size(...) bytes, 256-byte aligned.  After the
  * call the workspace holds the intermediates at the offsets reported by
- * oz2_workspace_layout (they stay valid until the workspace is reused). */
+ * oz2_workspace_layout (they stay valid until the workspace is reused).
+ * With OZ2_FLAG_FUSED, num_moduli 11 or 12 and k ≤ 256 (k padded to 256 or
+ * less) the residue GEMM and the reconstruction run fused; the residues
+ * region then holds that kernel's scratch instead of the residue matrices.
+ * The result C is the same either way, bit for bit. */
 int oz2_dgemm_ex(int64_t m, int64_t n, int64_t k,
                  const double* d_A, int64_t lda,
                  const double* d_B, int64_t ldb,
@@ -172,7 +184,9 @@ int oz2_dgemm_ex(int64_t m, int64_t n, int64_t k,
  *   residues              int16  r matrices C^(i), each m×n column-major
  *                                with ld = res_ld (matrix i starts at element
  *                                i·n·res_ld), centred in
- *                                [-⌊m_i/2⌋, m_i-1-⌊m_i/2⌋]
+ *                                [-⌊m_i/2⌋, m_i-1-⌊m_i/2⌋]; after a fused
+ *                                call (see oz2_dgemm_ex) the fused kernel's
+ *                                scratch instead
  */
 typedef struct {
   size_t ra, cb, row_flag, col_flag, d, e, urow, misc;

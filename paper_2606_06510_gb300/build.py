@@ -17,7 +17,7 @@ CSRC = os.path.join(HERE, "csrc")
 OBJ = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "liboz2.so")
 SOURCES = ["oz2_api.cu", "k_scan.cu", "k_deconstruct.cu", "k_gemm.cu", "k_crt.cu", "k_fallback.cu",
-           "oz2_noalloc.cu"]
+           "k_fused.cu", "oz2_noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
          "--expt-relaxed-constexpr", "-DNDEBUG"]

@@ -545,6 +545,10 @@ static int run_stages(int64_t m, int64_t n, int64_t k, const double* A, int64_t 
 
   const bool timing = (flags & OZ2_FLAG_TIMING) != 0;
   const bool simt = (flags & OZ2_FLAG_DEBUG_SIMT_GEMM) != 0;
+  // On request, for short k: the residue GEMM and the reconstruction fused,
+  // the residues kept on chip; the residue region then holds the fused
+  // kernel's list of outputs left to the exact reconstruction.
+  const bool fused = !simt && (flags & OZ2_FLAG_FUSED) != 0 && fused_crt_applies(L.k_pad, num_moduli);
   int dev = 0;
   cudaGetDevice(&dev);
   HostStats& hs = g_host_stats[dev];
@@ -598,14 +602,21 @@ static int run_stages(int64_t m, int64_t n, int64_t k, const double* A, int64_t 
     const int64_t cols = blocked ? blocks->widths[bi] : n;
     const uint8_t* pb0 = pb + static_cast<size_t>(c0 / kPlaneRows) * (L.k_pad / kPlaneLine) * L.num_planes *
                                   static_cast<size_t>(kPlaneBlock);
-    // The magnitude planes are dead once the scales are chosen: their region
-    // is the scratch for the partial residues of a split-K residue GEMM.
-    err = launch_plane_gemm(m, cols, L.k_pad, mods, pa, pb0, simt ? 2 : 0, res, L.res_ld, nullptr, ds->status, s,
-                            reinterpret_cast<int16_t*>(mag_a), L.planes_a - L.mag_a);
-    mark(6);
-    if (err == cudaSuccess)
-      err = launch_reconstruct(m, cols, mods, res, L.res_ld, d, e + c0, C + c0 * ldc, ldc, true, s);
-    mark(7);
+    if (fused) {
+      err = launch_fused_crt(m, cols, L.k_pad, mods, pa, pb0, d, e + c0, rf, cf + c0, C + c0 * ldc, ldc, res,
+                             L.total - L.residues, ds->status, s);
+      mark(6);
+      mark(7);
+    } else {
+      // The magnitude planes are dead once the scales are chosen: their region
+      // is the scratch for the partial residues of a split-K residue GEMM.
+      err = launch_plane_gemm(m, cols, L.k_pad, mods, pa, pb0, simt ? 2 : 0, res, L.res_ld, nullptr, ds->status, s,
+                              reinterpret_cast<int16_t*>(mag_a), L.planes_a - L.mag_a);
+      mark(6);
+      if (err == cudaSuccess)
+        err = launch_reconstruct(m, cols, mods, res, L.res_ld, d, e + c0, C + c0 * ldc, ldc, true, s);
+      mark(7);
+    }
     if (err == cudaSuccess)
       err = launch_fallback_lists(m, cols, k, A, lda, B + c0 * ldb, ldb, rf, cf + c0, misc, C + c0 * ldc, ldc, s,
                                   c0 > 0);

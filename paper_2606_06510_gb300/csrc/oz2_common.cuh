@@ -222,6 +222,15 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map
       : "memory");
 }
 
+// 2-D tiled TMA load into this CTA's shared memory, completing on an mbarrier.
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, uint32_t bar, int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4}], [%2];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(x), "r"(y)
+      : "memory");
+}
+
 __device__ __forceinline__ void prefetch_tensormap(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
 }
@@ -348,6 +357,12 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
         "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
       : "r"(taddr));
 }
+// 32 lanes × 32 bits, 8 consecutive columns per thread.
+__device__ __forceinline__ void tmem_ld8(uint32_t taddr, uint32_t (&v)[8]) {
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+               : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7])
+               : "r"(taddr));
+}
 // 32 lanes × 32 bits, 16 consecutive columns per thread.
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&v)[16]) {
   asm volatile(
@@ -449,6 +464,16 @@ cudaError_t launch_fallback_lists(int64_t m, int64_t n, int64_t k, const double*
                                   cudaStream_t st, bool zero_counts);
 // The tensor-pipe rate probe (k_gemm.cu); reports the CTA pairs it runs on.
 cudaError_t launch_mma_rate(int64_t iters, Oz2Device* dev, int* pairs_out, cudaStream_t st);
+// The fused residue GEMM and reconstruction (k_fused.cu) for r = 11, 12 and
+// k_pad ≤ kFusedMaxKPad: C from the digit planes, without residue matrices.
+// `scratch` (scratch_bytes, 16-byte aligned, at least 16 + 8·m·n bytes)
+// holds the list of outputs the fast reconstruction leaves.
+constexpr int64_t kFusedMaxKPad = 256;
+bool fused_crt_applies(int64_t k_pad, int r);
+cudaError_t launch_fused_crt(int64_t m, int64_t n, int64_t k_pad, const Oz2Moduli& mods, const uint8_t* planes_a,
+                             const uint8_t* planes_b, const int32_t* d, const int32_t* e, const uint8_t* row_flag,
+                             const uint8_t* col_flag, double* C, int64_t ldc, void* scratch, size_t scratch_bytes,
+                             Oz2Device* dev, cudaStream_t st);
 cudaError_t launch_native(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda,
                           const double* B, int64_t ldb, double* C, int64_t ldc, cudaStream_t st);
 }  // namespace oz2

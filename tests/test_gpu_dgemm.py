@@ -51,9 +51,12 @@ def test_small_workload_bit_exact_and_accurate(oz):
     assert np.array_equal(v["d"], res.d) and np.array_equal(v["e"], res.e)
     assert np.array_equal(v["residues"], res.residues)
     assert cref.scaled_error(C, A, B) <= 1e-15
-    # the production entry (own workspace) gives the same bits
+    # the production entry (own workspace) gives the same bits, and so does
+    # the fused residue GEMM and reconstruction
     C2 = oz.oz2_dgemm(to_dev(A), to_dev(B), num_moduli=12).cpu().numpy()
     assert_same(C2, res.C)
+    C3, _ = run_ex(oz, A, B, 12, flags=oz.FLAG_FUSED)
+    assert_same(C3, res.C)
 
 
 @pytest.mark.parametrize("shape", [(1, 1, 1), (100, 77, 333), (257, 129, 129), (64, 300, 7), (3, 5, 1000)])
@@ -73,6 +76,8 @@ def test_moduli_counts(oz, r):
     C, v = run_ex(oz, A, B, r)
     assert_same(C, res.C)
     assert np.array_equal(v["residues"], res.residues)
+    C, _ = run_ex(oz, A, B, r, flags=oz.FLAG_FUSED)   # fused for r = 11, 12 (k = 160)
+    assert_same(C, res.C)
 
 
 @pytest.mark.parametrize("quant", ["tz", "rn"])
