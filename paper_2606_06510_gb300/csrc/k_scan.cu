@@ -24,12 +24,13 @@ __device__ __forceinline__ int scan_key(double x) {
   return E - 1022 + 2048;
 }
 
-// Rows of column-major A: thread per row, grid.y splits k.
-__global__ void scan_a_kernel(int64_t m, int64_t k, const double* __restrict__ A, int64_t lda,
-                              int chunk, int* __restrict__ key) {
-  int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+// Rows of column-major A: thread per row, block row `by` of the k-chunks.
+__device__ __forceinline__ void scan_a_rows(int64_t bx, int64_t by, int64_t m, int64_t k,
+                                            const double* __restrict__ A, int64_t lda, int chunk,
+                                            int* __restrict__ key) {
+  int64_t i = bx * (int64_t)blockDim.x + threadIdx.x;
   if (i >= m) return;
-  int64_t l0 = (int64_t)blockIdx.y * chunk;
+  int64_t l0 = by * chunk;
   int64_t l1 = min(k, l0 + chunk);
   int best = 0;
   const double* p = A + i + l0 * lda;
@@ -42,14 +43,15 @@ __global__ void scan_a_kernel(int64_t m, int64_t k, const double* __restrict__ A
   if (best) atomicMax(key + i, best);
 }
 
-// Columns of column-major B: warp per column, lanes over l, grid.y splits k
-// into even-sized chunks; 16-byte loads when the column start is aligned.
-__global__ void scan_b_kernel(int64_t n, int64_t k, const double* __restrict__ B, int64_t ldb,
-                              int chunk, int vec, int* __restrict__ key) {
+// Columns of column-major B: warp per column, lanes over l, block row `by`
+// of the even-sized k-chunks; 16-byte loads when the column start is aligned.
+__device__ __forceinline__ void scan_b_cols(int64_t bx, int64_t by, int64_t n, int64_t k,
+                                            const double* __restrict__ B, int64_t ldb, int chunk, int vec,
+                                            int* __restrict__ key) {
   int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  int64_t j = blockIdx.x * (int64_t)(blockDim.x >> 5) + warp;
+  int64_t j = bx * (int64_t)(blockDim.x >> 5) + warp;
   if (j >= n) return;
-  int64_t l0 = (int64_t)blockIdx.y * chunk;
+  int64_t l0 = by * chunk;
   int64_t l1 = min(k, l0 + chunk);
   const double* col = B + j * ldb;
   int best = 0;
@@ -76,6 +78,25 @@ __global__ void scan_b_kernel(int64_t n, int64_t k, const double* __restrict__ B
   }
   best = __reduce_max_sync(0xffffffffu, best);
   if (lane == 0 && best) atomicMax(key + j, best);
+}
+
+// Both operands in one launch: blocks [0, ga) scan rows of A (gax blocks of
+// 256 rows per k-chunk), the rest scan columns of B (gbx blocks of 8 columns
+// per k-chunk).
+struct ScanGrid {
+  int64_t ga, gax, gbx;
+  int achunk, bchunk, vec;
+};
+__global__ void __launch_bounds__(256) scan_kernel(int64_t m, int64_t n, int64_t k, const double* __restrict__ A,
+                                                   int64_t lda, const double* __restrict__ B, int64_t ldb, ScanGrid g,
+                                                   int* __restrict__ ra, int* __restrict__ cb) {
+  const int64_t b = blockIdx.x;
+  if (b < g.ga) {
+    scan_a_rows(b % g.gax, b / g.gax, m, k, A, lda, g.achunk, ra);
+  } else {
+    const int64_t bb = b - g.ga;
+    scan_b_cols(bb % g.gbx, bb / g.gbx, n, k, B, ldb, g.bchunk, g.vec, cb);
+  }
 }
 
 // One block per operand (0: rows of A, 1: columns of B).  Decodes the scan
@@ -182,30 +203,28 @@ cudaError_t launch_scan(int64_t m, int64_t n, int64_t k, const double* A, int64_
   // The scan keys are maxima taken with atomics: zero unless the caller has.
   if (zero_keys && m > 0 && (err = cudaMemsetAsync(out.ra, 0, sizeof(int) * m, st)) != cudaSuccess) return err;
   if (zero_keys && n > 0 && (err = cudaMemsetAsync(out.cb, 0, sizeof(int) * n, st)) != cudaSuccess) return err;
-  if (k > 0) {
-    int chunk = 64;
-    int64_t ks = (k + chunk - 1) / chunk;
+  if (k > 0 && (m > 0 || n > 0)) {
+    ScanGrid g{};
+    g.achunk = 64;
+    int64_t ks = (k + g.achunk - 1) / g.achunk;
     if (ks > 65535) {
-      chunk = static_cast<int>((k + 65534) / 65535);
-      ks = (k + chunk - 1) / chunk;
+      g.achunk = static_cast<int>((k + 65534) / 65535);
+      ks = (k + g.achunk - 1) / g.achunk;
     }
-    if (m > 0) {
-      dim3 g(static_cast<unsigned>((m + 255) / 256), static_cast<unsigned>(ks));
-      count_launch();
-      scan_a_kernel<<<g, 256, 0, st>>>(m, k, A, lda, chunk, out.ra);
-    }
-    int bchunk = 1024;
-    int64_t bks = (k + bchunk - 1) / bchunk;
+    g.bchunk = 1024;
+    int64_t bks = (k + g.bchunk - 1) / g.bchunk;
     if (bks > 65535) {
-      bchunk = static_cast<int>((k + 65534) / 65535 + 1) & ~1;
-      bks = (k + bchunk - 1) / bchunk;
+      g.bchunk = static_cast<int>((k + 65534) / 65535 + 1) & ~1;
+      bks = (k + g.bchunk - 1) / g.bchunk;
     }
-    if (n > 0) {
-      const int vec = (ldb % 2 == 0) && (reinterpret_cast<uintptr_t>(B) % 16 == 0);
-      dim3 g(static_cast<unsigned>((n + 7) / 8), static_cast<unsigned>(bks));
-      count_launch();
-      scan_b_kernel<<<g, 256, 0, st>>>(n, k, B, ldb, bchunk, vec, out.cb);
-    }
+    g.gax = (m + 255) / 256;
+    g.ga = m > 0 ? g.gax * ks : 0;
+    g.gbx = (n + 7) / 8;
+    const int64_t gb = n > 0 ? g.gbx * bks : 0;
+    g.vec = (ldb % 2 == 0) && (reinterpret_cast<uintptr_t>(B) % 16 == 0);
+    if (g.ga + gb > 0x7FFFFFFFLL) return cudaErrorInvalidValue;
+    count_launch();
+    scan_kernel<<<static_cast<unsigned>(g.ga + gb), 256, 0, st>>>(m, n, k, A, lda, B, ldb, g, out.ra, out.cb);
   }
   count_launch();
   finalize_flags_kernel<<<2, kFinalizeThreads, 0, st>>>(m, n, out.ra, out.cb, out.row_flag, out.col_flag,

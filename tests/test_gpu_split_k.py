@@ -18,11 +18,12 @@ pytestmark = pytest.mark.gpu
 
 
 def unsplit_launches(m):
-    """Kernels of an unsplit call: prepare, 3 scan, magnitude, "+1", scales,
-    deconstruct, GEMM, CRT, 2 fallback.  (C here has ld = m: for even m the
-    CRT takes every row in pairs, for odd m it runs the element-wise
-    instance alone, so it is one launch either way.)"""
-    return 12
+    """Kernels of an unsplit call: prepare, 2 scan (A and B in one launch,
+    then the flags), magnitude, "+1", scales, deconstruct, GEMM, CRT, 2
+    fallback.  (C here has ld = m: for even m the CRT takes every row in
+    pairs, for odd m it runs the element-wise instance alone, so it is one
+    launch either way.)"""
+    return 11
 
 
 @pytest.fixture(scope="module")

@@ -100,12 +100,12 @@ def test_split_k_in_the_scratch_then_an_unsplit_call(env, shape, r, parts):
     B = to_dev(wl.random_matrix(k, n, 1.0, 5252 + r))
     oz.oz2_get_stats()                      # resets the launch counter
     got = call_noalloc(env, A, B, r)
-    assert oz.oz2_get_stats()["kernel_launches"] == 13
+    assert oz.oz2_get_stats()["kernel_launches"] == 12
     want = oz.oz2_dgemm(A, B, num_moduli=r).cpu().numpy()
     assert np.array_equal(got, want)
     A2 = to_dev(wl.random_matrix(96, 300, 0.5, 5353 + r))
     B2 = to_dev(wl.random_matrix(300, 80, 0.5, 5454 + r))
     oz.oz2_get_stats()
     got2 = call_noalloc(env, A2, B2, r)
-    assert oz.oz2_get_stats()["kernel_launches"] == 12
+    assert oz.oz2_get_stats()["kernel_launches"] == 11
     assert np.array_equal(got2, oz.oz2_dgemm(A2, B2, num_moduli=r).cpu().numpy())
