@@ -17,14 +17,17 @@
 // modulus) and one 16-byte store of its two results (a warp writes 512
 // contiguous bytes), with no transposition.  Each thread walks a strided
 // set of columns and loads the next column's residues while it computes the
-// current one.  An output that the fast path leaves is marked with a NaN
-// sentinel and recomputed after the loop, which keeps the exact paths'
-// register footprint out of the loop.
+// current one.  An output that the fast path leaves is recorded in a short
+// per-thread list (local memory, touched only then) and recomputed after the
+// loop, which keeps the exact paths' registers out of the loop; past the
+// list's length the output is marked with a NaN sentinel and found again by
+// a rescan of the thread's later columns.
 #include "oz2_crt.cuh"
 
 namespace oz2 {
 
 constexpr int kCrtThreads = 256;
+constexpr int kCrtFailSlots = 8;  // outputs per thread the fast path may leave before a rescan
 
 // Resident blocks per SM the register budget is sized for: the two-word
 // path fits 64 registers (four blocks) up to r = 12 in the FAST kernel and
@@ -39,12 +42,13 @@ constexpr int crt_min_blocks() {
 // column's residues are loaded while the previous column is reconstructed,
 // alternating between two buffers.  FAST: both rows present, 4-byte residue
 // loads and 16-byte stores possible; otherwise element-wise accesses.
-// Returns how many outputs were left to Garner's algorithm.
+// Outputs the fast path leaves go into `fails` as 2·(column iteration) + row
+// (0 or 1), the first kCrtFailSlots of them; returns how many there were.
 template <int R, bool FAST>
-__device__ __forceinline__ uint32_t crt_columns(int64_t n, int64_t row, bool pair, int d0, int d1,
-                                                const Oz2Moduli& mods, unsigned long long err,
-                                                const int16_t* __restrict__ res, int64_t ldr,
-                                                const int* __restrict__ e, double* cbase, int64_t ldc) {
+__device__ __forceinline__ int crt_columns(int64_t n, int64_t row, bool pair, int d0, int d1, const Oz2Moduli& mods,
+                                           unsigned long long err, const int16_t* __restrict__ res, int64_t ldr,
+                                           const int* __restrict__ e, double* cbase, int64_t ldc,
+                                           int (&fails)[kCrtFailSlots]) {
   const int64_t step = gridDim.y;
   const int64_t off_step = step * ldr;
   // Residue matrix k starts at res + k·mstride (the same for every thread,
@@ -65,9 +69,7 @@ __device__ __forceinline__ uint32_t crt_columns(int64_t n, int64_t row, bool pai
         w[k] = static_cast<uint16_t>(base[k][off]) | (pair ? static_cast<uint32_t>(base[k][off + 1]) << 16 : 0u);
     }
   };
-  // Bit j: the j-th column of this thread has an output left to the exact
-  // path (bit 31: one of the 32nd or later columns has).
-  uint32_t pending = 0;
+  int nfail = 0;
   int iter = 0;
   auto column = [&](const uint32_t (&w)[R], int ec, int64_t col) {
     double v[2];
@@ -80,7 +82,8 @@ __device__ __forceinline__ uint32_t crt_columns(int64_t n, int64_t row, bool pai
       double val;
       if (!crt_fast<R>(c, -((u ? d1 : d0) + ec), mods, err, val)) {
         val = __longlong_as_double(kCrtSentinel);
-        pending |= 1u << (iter < 31 ? iter : 31);
+        if (nfail < kCrtFailSlots) fails[nfail] = 2 * iter + u;
+        ++nfail;
       }
       v[u] = val;
     }
@@ -117,7 +120,7 @@ __device__ __forceinline__ uint32_t crt_columns(int64_t n, int64_t row, bool pai
     col += step;
     off += off_step;
   }
-  return pending;
+  return nfail;
 }
 
 // Rows [row0, row0 + rows) of C.  FAST kernels take row pairs with 4-byte
@@ -135,27 +138,25 @@ __global__ void __launch_bounds__(kCrtThreads, crt_min_blocks<R, FAST>())
   const bool pair = rel + 1 < rows;
   const int d0 = d[row], d1 = pair ? d[row + 1] : 0;
   double* cbase = C + row;
-  uint32_t pending = crt_columns<R, FAST>(n, row, pair, d0, d1, mods, err, res, ldr, e, cbase, ldc);
-  if (pending == 0) return;
-  // Outputs the fast path left to the exact paths (this thread's own): the
-  // columns its mask marks, and every column from the 32nd on if bit 31 is set.
+  int fails[kCrtFailSlots];
+  const int nfail = crt_columns<R, FAST>(n, row, pair, d0, d1, mods, err, res, ldr, e, cbase, ldc, fails);
+  if (nfail == 0) return;
+  // Outputs the fast path left to the exact paths (this thread's own).
   const int64_t step = gridDim.y;
-  const int64_t tail = blockIdx.y + 31 * step;
-  while (pending) {
-    const int j = __ffs(pending) - 1;
-    pending &= pending - 1;
-    const int64_t c_lo = blockIdx.y + j * step;
-    const int64_t c_hi = j < 31 ? c_lo + 1 : n;
-    for (int64_t col = j < 31 ? c_lo : tail; col < c_hi && col < n; col += (j < 31 ? 1 : step)) {
-      for (int u = 0; u < (pair ? 2 : 1); ++u) {
-        double* q = cbase + col * ldc + u;
-        if (__double_as_longlong(*q) != kCrtSentinel) continue;
-        int c[R];
+  auto exact = [&](int64_t col, int u) {
+    int c[R];
 #pragma unroll
-        for (int k = 0; k < R; ++k) c[k] = res[(k * n + col) * ldr + row + u];
-        *q = crt_exact<R>(c, -((u ? d1 : d0) + __ldg(e + col)), mods);
-      }
-    }
+    for (int k = 0; k < R; ++k) c[k] = res[(k * n + col) * ldr + row + u];
+    cbase[col * ldc + u] = crt_exact<R>(c, -((u ? d1 : d0) + __ldg(e + col)), mods);
+  };
+  const int listed = nfail < kCrtFailSlots ? nfail : kCrtFailSlots;
+  for (int i = 0; i < listed; ++i) exact(blockIdx.y + (fails[i] >> 1) * step, fails[i] & 1);
+  if (nfail > kCrtFailSlots) {
+    // More than the list holds: the rest carry the sentinel, from the column
+    // of the last one listed on (whose other row may be one of them).
+    for (int64_t col = blockIdx.y + (fails[kCrtFailSlots - 1] >> 1) * step; col < n; col += step)
+      for (int u = 0; u < (pair ? 2 : 1); ++u)
+        if (__double_as_longlong(cbase[col * ldc + u]) == kCrtSentinel) exact(col, u);
   }
 }
 

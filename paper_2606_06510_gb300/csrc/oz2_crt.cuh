@@ -378,6 +378,15 @@ __device__ __forceinline__ bool crt_value_y96(const int (&c)[R], int E, const Oz
   Y96 y{0, 0, 0u};
 #pragma unroll
   for (int k = 0; k < R; ++k) y96_add(y, c[k], mods, k);
+  if ((y.a0 | y.a1 | static_cast<long long>(y.a2)) == 0) {
+    // Y = 0: X is 0 when every residue is (rows and columns that are zero in
+    // the emulation), whose result is +0; any other X takes the exact path.
+    int any = 0;
+#pragma unroll
+    for (int k = 0; k < R; ++k) any |= c[k];
+    out = 0.0;
+    return any == 0;
+  }
   return y96_finish(y, E, mods, err, out);
 }
 

@@ -63,6 +63,8 @@ def fast_path(c, E, r, err):
     a1 = sum(ck * f1 for ck, (_, _, _, _, f1, _) in zip(c, ks))
     a2 = sum(ck * f2 for ck, (_, _, _, _, _, f2) in zip(c, ks)) & MASK32
     assert -2 ** 63 <= a0 < 2 ** 63 and -2 ** 63 <= a1 < 2 ** 63
+    if a0 == 0 and a1 == 0 and a2 == 0:      # Y = 0: X = 0 when every residue is
+        return 0.0 if not any(c) else None
     s1 = (a0 >> 32) + a1
     w0, w1 = a0 & MASK32, s1 & MASK32
     w2 = ((s1 >> 32) + a2) & MASK32
@@ -186,7 +188,8 @@ def test_small_and_subnormal_results_defer():
     r = 12
     M, mods, _ = constants(r)
     err = err_bound(M, mods, True)
-    for x in (0, 5, -(2 ** 40), 2 ** 80):
+    assert fast_path(residues(0, mods), -10, r, err) == 0.0      # all residues zero: +0
+    for x in (5, -(2 ** 40), 2 ** 80):
         assert fast_path(residues(x, mods), -10, r, err) is None
     x = 2 ** 100 + 12345
     assert fast_path(residues(x, mods), -1200, r, err) is None      # subnormal result

@@ -214,6 +214,80 @@ def test_reconstruct(oz):
                 assert C[i, j] == want and np.signbit(C[i, j]) == np.signbit(want), (r, m, n, i, j)
 
 
+@pytest.mark.parametrize("r,m,n,ldr,ldc,c_off", [
+    (12, 1100, 5, 1104, 1100, 0),    # several row blocks, the last ragged
+    (12, 1031, 4, 1040, 1032, 0),    # odd m: the last row runs in the element-wise kernel
+    (16, 600, 3, 608, 600, 0),       # five-limb path
+    (6, 8, 1, 8, 8, 0),              # one short column
+    (11, 300, 4, 304, 300, 1),       # C not 16-byte aligned: element-wise kernel
+    (12, 64, 3, 64, 65, 0),          # odd ldc: element-wise kernel
+])
+def test_reconstruct_tiles_and_alignment(oz, r, m, n, ldr, ldc, c_off):
+    """The row-pair kernel on ragged row blocks and an odd last row, and the
+    element-wise kernel for buffers the row-pair one cannot take, against
+    Garner's algorithm in the oracle; rows of C beyond m stay untouched."""
+    import torch
+    rng = np.random.default_rng(1000 + m)
+    mods = orc.moduli(r)
+    R = np.stack([orc.centred(rng.integers(0, mi, size=(m, n)), mi) for mi in mods])
+    R[:, :7, 0] = 0                                    # X = 0 for a few outputs
+    d = rng.integers(40, 80, size=m)
+    e = rng.integers(40, 80, size=n)
+    d[1], d[2], d[3] = 1100, 1180, -1100               # subnormal, underflow, overflow rows
+    buf = torch.full((r, n, ldr), 777, dtype=torch.int16)
+    buf[:, :, :m] = torch.from_numpy(R.transpose(0, 2, 1).astype(np.int16))
+    res = buf.cuda()[:, :, :m].transpose(1, 2)
+    cbuf = torch.full((n * ldc + c_off,), 12345.0, dtype=torch.float64, device="cuda")
+    C = cbuf[c_off:].view(n, ldc).t()[:m, :]
+    oz.oz2_reconstruct(res, torch.from_numpy(d.astype(np.int32)).cuda(), torch.from_numpy(e.astype(np.int32)).cuda(),
+                       m, n, r, C=C)
+    got = C.cpu().numpy()
+    X = orc.garner_value(R, mods)
+    for i in range(m):
+        for j in range(n):
+            want = orc.unscale_one(int(X[i, j]), -int(d[i]) - int(e[j]))
+            assert got[i, j] == want and np.signbit(got[i, j]) == np.signbit(want), (r, m, n, i, j)
+    # rows beyond m of each column of C are untouched
+    full = cbuf[c_off:].view(n, ldc).cpu().numpy()
+    assert (full[:, m:] == 12345.0).all()
+
+
+def test_reconstruct_many_outputs_left_to_the_exact_path(oz):
+    """Two rows and more columns than the launch has column strides, so each
+    thread walks about ten columns, with most outputs small (|X| < 2^80),
+    which the 96-bit fast path of r = 12 leaves to the exact path: threads
+    leave more outputs than their list holds and find the rest again by
+    rescanning; large, zero and midpoint-free outputs are mixed in."""
+    import random
+    import torch
+    r = 12
+    mods = orc.moduli(r)
+    M = orc.modulus_product(mods)
+    rng = random.Random(77)
+    m, n = 2, 12500
+    xs = []
+    for _ in range(m * n):
+        t = rng.random()
+        if t < 0.7:
+            xs.append(rng.randrange(-(1 << 80), 1 << 80))
+        elif t < 0.8:
+            xs.append(0)
+        else:
+            xs.append(rng.randrange(-(M // 4), M // 4))
+    X = np.array(xs, dtype=object).reshape(m, n)
+    R = np.zeros((r, m, n), dtype=np.int64)
+    for k, mk in enumerate(mods):
+        R[k] = np.vectorize(lambda x: int(orc.centred(x % mk, mk)), otypes=[np.int64])(X)
+    d = np.array([3, -40], dtype=np.int64)
+    e = np.array([rng.randrange(-60, 60) for _ in range(n)], dtype=np.int64)
+    C = oz.oz2_reconstruct(torch.from_numpy(R.astype(np.int16)).cuda(), torch.from_numpy(d.astype(np.int32)).cuda(),
+                           torch.from_numpy(e.astype(np.int32)).cuda(), m, n, r).cpu().numpy()
+    for i in range(m):
+        for j in range(n):
+            want = orc.unscale_one(int(X[i, j]), -int(d[i]) - int(e[j]))
+            assert C[i, j] == want and np.signbit(C[i, j]) == np.signbit(want), (i, j)
+
+
 def test_reconstruct_near_the_range_boundary(oz):
     """Integers at and next to ±M/2, where the fast reconstruction defers to
     Garner's algorithm, and a band of values around them."""
