@@ -71,6 +71,15 @@ typedef enum { OZ2_SCALE_R2 = 0, OZ2_SCALE_R1 = 1 } oz2_scale_mode;
  * A through L2 once per 32 columns of C, and on one GB300 it measured slower
  * than the two launches for every shape tried; see oz2_dgemm_ex. */
 #define OZ2_FLAG_FUSED       0x4u
+/* For a skinny C (n ≤ 32, m ≥ 128, k padded to 1024 or more): form A's
+ * digit planes on chip from A inside the residue GEMM (plane storage mode F,
+ * §"plane-storage modes"), so they are never written to device memory and
+ * read back, instead of storing them.  It moves fewer DRAM bytes but runs
+ * the conversion on one CTA per 128 rows of A; on one GB300 the batched
+ * GEMV 16384 × 16 × 16384 took 5.12 ms this way against 4.55 ms with the
+ * planes stored, so it is not the default.  Ignored where it does not
+ * apply; see oz2_dgemm_ex. */
+#define OZ2_FLAG_ON_THE_FLY  0x8u
 /* Diagnostic only: run the "+1" and residue plane GEMMs on CUDA cores with
  * the same integer plane products and epilogue arithmetic (slow; used by
  * the tests to separate tensor-core issues from the rest of the path). */
@@ -161,7 +170,10 @@ size_t oz2_workspace_size(int64_t m, int64_t n, int64_t k, int num_moduli);
  * With OZ2_FLAG_FUSED, num_moduli 11 or 12 and k ≤ 256 (k padded to 256 or
  * less) the residue GEMM and the reconstruction run fused; the residues
  * region then holds that kernel's scratch instead of the residue matrices.
- * The result C is the same either way, bit for bit. */
+ * With OZ2_FLAG_ON_THE_FLY and a skinny C (n ≤ 32, m ≥ 128, k padded to
+ * 1024 or more) A's digit planes are formed on chip from A inside the
+ * residue GEMM and never stored (the planes_a region is then left
+ * unwritten).  The result C is the same on every path, bit for bit. */
 int oz2_dgemm_ex(int64_t m, int64_t n, int64_t k,
                  const double* d_A, int64_t lda,
                  const double* d_B, int64_t ldb,

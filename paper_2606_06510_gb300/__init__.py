@@ -26,6 +26,7 @@ SCALE = {"r2": 0, "r1": 1}
 FLAG_NO_FALLBACK = 0x1
 FLAG_TIMING = 0x2
 FLAG_FUSED = 0x4
+FLAG_ON_THE_FLY = 0x8
 FLAG_DEBUG_SIMT_GEMM = 0x100
 STAGES = ("scan", "magnitude", "plus_one_gemm", "scale", "deconstruct", "residue_gemm", "crt", "fallback")
 

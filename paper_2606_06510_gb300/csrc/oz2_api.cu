@@ -302,7 +302,7 @@ static int device_state(DeviceState** out) {
         const int m = kModuliAll[i];
         if (isqrt_exact(m)) continue;  // square moduli compute their digits
         for (int j = 0; j < 2 * m; ++j) {
-          const int r = floor_mod(j - kDecBias % m, m);
+          const int r = floor_mod(j - static_cast<int>(kDecBias % static_cast<uint32_t>(m)), m);
           const int d = r > m - 1 - m / 2 ? r - m : r;  // centred residue
           const uint32_t w = plane_word(d, m, t == 0);
           if (w == 0xFFFFFFFFu) return OZ2_ERR_CUDA;
@@ -549,6 +549,9 @@ static int run_stages(int64_t m, int64_t n, int64_t k, const double* A, int64_t 
   // the residues kept on chip; the residue region then holds the fused
   // kernel's list of outputs left to the exact reconstruction.
   const bool fused = !simt && (flags & OZ2_FLAG_FUSED) != 0 && fused_crt_applies(L.k_pad, num_moduli);
+  // A skinny C: A's digit planes formed on chip inside the residue GEMM
+  // (never stored), only B deconstructed ahead.
+  const bool onfly = !simt && !fused && (flags & OZ2_FLAG_ON_THE_FLY) != 0 && modef_applies(m, n, L.k_pad);
   int dev = 0;
   cudaGetDevice(&dev);
   HostStats& hs = g_host_stats[dev];
@@ -592,7 +595,8 @@ static int run_stages(int64_t m, int64_t n, int64_t k, const double* A, int64_t 
   if (err == cudaSuccess) err = launch_choose_scales(m, n, k, mods, scale, urow, ra, cb, rf, cf, d, e, ds->status, s);
   mark(4);
   if (err == cudaSuccess)
-    err = launch_deconstruct(m, n, k, mods, ds->table_a, ds->table_b, A, lda, B, ldb, d, e, rf, cf, quant, pa, pb, s);
+    err = launch_deconstruct(onfly ? 0 : m, n, k, mods, ds->table_a, ds->table_b, A, lda, B, ldb, d, e, rf, cf, quant,
+                             pa, pb, s);
   mark(5);
   // Phase 2 by column blocks (stage timing needs a single block).
   const bool blocked = blocks && blocks->count > 1 && !ts;
@@ -608,10 +612,14 @@ static int run_stages(int64_t m, int64_t n, int64_t k, const double* A, int64_t 
       mark(6);
       mark(7);
     } else {
-      // The magnitude planes are dead once the scales are chosen: their region
-      // is the scratch for the partial residues of a split-K residue GEMM.
-      err = launch_plane_gemm(m, cols, L.k_pad, mods, pa, pb0, simt ? 2 : 0, res, L.res_ld, nullptr, ds->status, s,
-                              reinterpret_cast<int16_t*>(mag_a), L.planes_a - L.mag_a);
+      if (onfly) {
+        err = launch_modef(m, cols, k, mods, ds->table_a, A, lda, d, rf, quant, pb0, res, L.res_ld, ds->status, s);
+      } else {
+        // The magnitude planes are dead once the scales are chosen: their
+        // region is the scratch for the partial residues of a split-K GEMM.
+        err = launch_plane_gemm(m, cols, L.k_pad, mods, pa, pb0, simt ? 2 : 0, res, L.res_ld, nullptr, ds->status, s,
+                                reinterpret_cast<int16_t*>(mag_a), L.planes_a - L.mag_a);
+      }
       mark(6);
       if (err == cudaSuccess)
         err = launch_reconstruct(m, cols, mods, res, L.res_ld, d, e + c0, C + c0 * ldc, ldc, true, s);

@@ -31,19 +31,26 @@ constexpr int kKSlabMerged = 4096;
 constexpr int kModuliList[kMaxModuli] = {1089, 1024, 961, 841, 625, 529, 511, 509,
                                          503,  499,  491, 487, 479, 467, 463, 461};
 
-// The deconstruction's digit-plane table holds 2m entries per nonsquare
+// The deconstruction splits each integer entry Ã (|Ã| < 2^62) into 21-bit
+// limbs, Ã = v0 + v1·2^21 + v2·2^42 with v0, v1 ∈ [0, 2^21) and v2 signed
+// (|v2| ≤ 2^20), and forms per modulus the 32-bit sum
+// Y = (v0 + kDecBias) + v1·c1 + v2·c2 ≡ Ã + kDecBias (mod m), with the
+// centred limb weights c1 = 2^21 mod m and c2 = 2^42 mod m (|c| ≤ 544).
+// kDecBias = 2^31 keeps Y inside (0, 2^32): |v1·c1| < 2^30.1 and
+// |v2·c2| < 2^29.1.  The digit-plane table holds 2m entries per nonsquare
 // modulus (entry i: the planes of the residue (i - kDecBias) mod m), so that
-// a quotient one too large, and the bias that keeps the residue sum
-// positive, cost nothing at the lookup.  Square moduli compute their digits.
-constexpr int kDecBias = 1 << 25;
+// a quotient one too large, and the bias, cost nothing at the lookup.
+// Square moduli compute their digits.
+constexpr uint32_t kDecBias = 1u << 31;
+constexpr int kLimbBits = 21;
 
 struct ModConst {
   int m;
   int s;          // square base, 0 for nonsquare moduli
   int plane_off;  // first plane of this modulus
   int table_off;  // nonsquare: first of its 2m entries in the digit-plane table
-  uint32_t limb1, limb2, limb3;  // 4·(2^16 mod m), 4·(2^32 mod m), 4·(2^48 mod m)
-  uint32_t magic;                // ⌈2^30/m⌉
+  int c1, c2;     // centred 2^21 mod m and 2^42 mod m
+  uint32_t magic; // ⌈2^32/m⌉
   // Square moduli (digits computed, not looked up): E = (⌊m/2⌋ - kDecBias)
   // mod m, the digit offsets h0 = ⌊s/2⌋ and h1 = ⌈(⌊m/2⌋ - h0)/s⌉, and
   // ⌈2^32/s⌉.
@@ -51,6 +58,12 @@ struct ModConst {
   int sq_h0, sq_h1;
   uint32_t sq_magic;
 };
+
+// x mod m in [-⌊m/2⌋, m - 1 - ⌊m/2⌋] (the centred residue) for x ≥ 0.
+constexpr int ce_centred(unsigned long long x, int m) {
+  const int r = static_cast<int>(x % static_cast<unsigned long long>(m));
+  return r > m - 1 - m / 2 ? r - m : r;
+}
 
 constexpr int ce_isqrt(int m) {
   int s = 0;
@@ -90,13 +103,12 @@ constexpr ModConst mod_const(int i) {
   c.plane_off = plane;
   c.table_off = 2 * toff;
   const unsigned long long um = static_cast<unsigned long long>(m);
-  c.limb1 = static_cast<uint32_t>(4 * ((1ull << 16) % um));
-  c.limb2 = static_cast<uint32_t>(4 * ((1ull << 32) % um));
-  c.limb3 = static_cast<uint32_t>(4 * ((1ull << 48) % um));
-  c.magic = static_cast<uint32_t>(((1ull << 30) + um - 1) / um);
+  c.c1 = ce_centred(1ull << kLimbBits, m);
+  c.c2 = ce_centred(1ull << (2 * kLimbBits), m);
+  c.magic = static_cast<uint32_t>(((1ull << 32) + um - 1) / um);
   if (c.s) {
     const int H = m / 2;
-    c.sq_e = static_cast<uint32_t>(((H - kDecBias) % m + m) % m);
+    c.sq_e = static_cast<uint32_t>((static_cast<long long>(H) - kDecBias % um + m) % m);
     c.sq_h0 = c.s / 2;
     c.sq_h1 = (H - c.sq_h0 + c.s - 1) / c.s;
     c.sq_magic = static_cast<uint32_t>(((1ull << 32) + c.s - 1) / static_cast<unsigned long long>(c.s));
@@ -357,6 +369,18 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
         "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
       : "r"(taddr));
 }
+// 32 lanes × 32 bits, 4 consecutive columns per thread.
+__device__ __forceinline__ void tmem_ld4(uint32_t taddr, uint32_t (&v)[4]) {
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3])
+               : "r"(taddr));
+}
+// 32 lanes × 32 bits, 4 consecutive columns per thread, stored.
+__device__ __forceinline__ void tmem_st4(uint32_t taddr, const uint32_t (&v)[4]) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1,%2,%3,%4};" ::"r"(taddr), "r"(v[0]), "r"(v[1]),
+               "r"(v[2]), "r"(v[3])
+               : "memory");
+}
 // 32 lanes × 32 bits, 8 consecutive columns per thread.
 __device__ __forceinline__ void tmem_ld8(uint32_t taddr, uint32_t (&v)[8]) {
   asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
@@ -400,6 +424,21 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr) {
   d |= static_cast<uint64_t>(1024u >> 4) << 32;
   d |= static_cast<uint64_t>(1u) << 46;
   d |= static_cast<uint64_t>(2u) << 61;
+  return d;
+}
+
+// Shared-memory matrix descriptor for a K-major operand tile without
+// swizzle: 8-row × 16-byte core matrices, each stored as 128 contiguous
+// bytes; `lbo` is the byte distance between core matrices adjacent in K and
+// `sbo` between core matrices adjacent in M (or N).  Start address >> 4 in
+// bits [0,14), LBO >> 4 in [16,30), SBO >> 4 in [32,46), descriptor version
+// 1 in [46,48), layout SWIZZLE_NONE (0) in [61,64).
+__device__ __forceinline__ uint64_t smem_desc_plain(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr >> 4) & 0x3FFFu);
+  d |= static_cast<uint64_t>((lbo >> 4) & 0x3FFFu) << 16;
+  d |= static_cast<uint64_t>((sbo >> 4) & 0x3FFFu) << 32;
+  d |= static_cast<uint64_t>(1u) << 46;
   return d;
 }
 
@@ -474,6 +513,15 @@ cudaError_t launch_fused_crt(int64_t m, int64_t n, int64_t k_pad, const Oz2Modul
                              const uint8_t* planes_b, const int32_t* d, const int32_t* e, const uint8_t* row_flag,
                              const uint8_t* col_flag, double* C, int64_t ldc, void* scratch, size_t scratch_bytes,
                              Oz2Device* dev, cudaStream_t st);
+// On-the-fly residues (k_deconstruct.cu): the residue GEMM of a skinny C
+// (n ≤ kModeFMaxN) with A's digit planes formed in shared memory from A
+// itself, never stored; B's planes come from the deconstruction.  Writes the
+// residue matrices as the residue GEMM does.
+constexpr int64_t kModeFMaxN = 32;
+bool modef_applies(int64_t m, int64_t n, int64_t k_pad);
+cudaError_t launch_modef(int64_t m, int64_t n, int64_t k, const Oz2Moduli& mods, const uint32_t* table_a,
+                         const double* A, int64_t lda, const int32_t* d, const uint8_t* row_flag, int quant,
+                         const uint8_t* planes_b, int16_t* residues, int64_t ldr, Oz2Device* dev, cudaStream_t st);
 cudaError_t launch_native(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda,
                           const double* B, int64_t ldb, double* C, int64_t ldc, cudaStream_t st);
 }  // namespace oz2

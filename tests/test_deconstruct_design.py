@@ -6,11 +6,11 @@ each entry's centred residues with 32-bit integer steps:
 * a branch-free truncating quantisation: the significand shifted up by 10
   and back down with clamping funnel shifts, the sign applied as a two's
   complement, for scales d ≤ 1083 (and d = -4096 for rows that are zero);
-* Ã split into three 16-bit limbs and a signed top limb, the lowest biased
-  by 2^25, summed per modulus with the limb weights 2^16j mod m pre-scaled
-  by 4;
-* a multiply-high quotient by ⌈2^30/m⌉ that may be one too large, so the
-  remainder lies in [-4m, 4m) and indexes a table of 2m entries rotated by
+* Ã split into 21-bit limbs, Ã = v0 + v1·2^21 + v2·2^42 with v2 signed,
+  the lowest biased by 2^31, summed per modulus with the centred limb
+  weights 2^21 mod m and 2^42 mod m, so the sum lies in (0, 2^32);
+* a multiply-high quotient by ⌈2^32/m⌉ that may be one too large, so the
+  remainder lies in [-m, m) and indexes a table of 2m entries rotated by
   the bias (nonsquare moduli);
 * for square moduli, an added constant that makes the remainder the centred
   residue plus ⌊m/2⌋, then balanced base-s digits by a multiply-high.
@@ -25,7 +25,8 @@ import pytest
 from oracle import ozaki2 as orc
 
 M32 = np.uint64(0xFFFFFFFF)
-BIAS = 1 << 25          # the limb-sum bias
+BIAS = 1 << 31          # the limb-sum bias
+LIMB = 21               # limb width
 TZ_FAST_MAX_D = 1083    # largest scale the branch-free path takes
 
 
@@ -39,8 +40,18 @@ def funnel_right_clamped(lo, hi, sh):
     return ((hi << np.uint64(32)) | lo) >> s & M32
 
 
+def split_word(tl, th):
+    """The kernel's limbs (w0, w1, w2) of the two's complement word th:tl
+    (tl unsigned 32-bit, th signed)."""
+    mask = np.uint64((1 << LIMB) - 1)
+    w0 = (tl & mask) | np.uint64(BIAS)
+    w1 = ((u64(th & 0xFFFFFFFF) << np.uint64(32) | tl) >> np.uint64(LIMB)) & mask
+    w2 = np.asarray(th, dtype=np.int64) >> (2 * LIMB - 32)
+    return w0, w1, w2
+
+
 def quantise_tz_limbs(x, d):
-    """The kernel's limbs (b, u1, u2, u3) of trunc(x·2^d)."""
+    """The kernel's limbs of trunc(x·2^d)."""
     bits = np.asarray(x, dtype=np.float64).view(np.uint64)
     hi, lo = bits >> np.uint64(32), bits & M32
     E = ((hi >> np.uint64(20)) & np.uint64(0x7FF)).astype(np.int64)
@@ -60,31 +71,29 @@ def quantise_tz_limbs(x, d):
     tl = t & M32
     th = (t >> np.uint64(32)).astype(np.int64)
     th = np.where(th >= 1 << 31, th - (1 << 32), th)
-    b = ((tl << np.uint64(2)) & np.uint64(0x3FFFC)) | np.uint64(4 * BIAS)
-    return b, tl >> np.uint64(16), u64(th & 0xFFFF), th >> 16
+    return split_word(tl, th)
 
 
 def limbs_of(At):
     """The same limbs taken straight from Ã (|Ã| < 2^62)."""
     At = np.asarray(At, dtype=np.int64)
-    tl = u64(At & 0xFFFFFFFF)
-    th = At >> 32
-    b = ((tl & np.uint64(0xFFFF)) << np.uint64(2)) | np.uint64(4 * BIAS)
-    return b, tl >> np.uint64(16), u64(th & 0xFFFF), th >> 16
+    return split_word(u64(At & 0xFFFFFFFF), At >> 32)
 
 
-def value_of(b, u1, u2, u3):
-    u0 = (b >> np.uint64(2)).astype(np.int64) - BIAS
-    return u0 + (u1.astype(np.int64) << 16) + (u2.astype(np.int64) << 32) + (u3 << 48)
+def value_of(w0, w1, w2):
+    return (w0.astype(np.int64) - BIAS) + (w1.astype(np.int64) << LIMB) + (w2 << (2 * LIMB))
 
 
-def limb_sum(b, u1, u2, u3, m, extra=0):
-    """Y = b + 4·extra + Σ u_j·4(2^16j mod m), wrapped to 32 bits, and the
-    same sum without wrapping."""
-    w = [4 * (pow(2, 16 * j, m)) for j in (1, 2, 3)]
-    exact = b.astype(np.int64) + 4 * extra + u1.astype(np.int64) * w[0] + u2.astype(np.int64) * w[1] + u3 * w[2]
-    Y = (b + np.uint64(4 * extra) + u1 * np.uint64(w[0]) + u2 * np.uint64(w[1])
-         + u64(u3 & 0xFFFFFFFF) * np.uint64(w[2])) & M32
+def centred_weight(j, m):
+    return int(orc.centred(pow(2, LIMB * j, m), m))
+
+
+def limb_sum(w0, w1, w2, m, extra=0):
+    """Y = w0 + extra + w1·c1 + w2·c2 with the centred weights c_j = 2^21j
+    mod m, wrapped to 32 bits, and the same sum without wrapping."""
+    c1, c2 = centred_weight(1, m), centred_weight(2, m)
+    exact = w0.astype(np.int64) + extra + w1.astype(np.int64) * c1 + w2 * c2
+    Y = (w0 + np.uint64(extra) + w1 * np.uint64(c1 & 0xFFFFFFFF) + u64(w2 & 0xFFFFFFFF) * np.uint64(c2 & 0xFFFFFFFF)) & M32
     return Y, exact
 
 
@@ -129,20 +138,31 @@ def test_limb_split_round_trip():
 
 @pytest.mark.parametrize("m", [m for m in orc.moduli(16) if not orc.square_base(m)])
 def test_nonsquare_table_index(m):
-    """Y - 4qm lies in [-4m, 4m), and entry m + (Y - 4qm)/4 of the rotated
-    table (entry i: the residue (i - 2^25) mod m) is Ã mod m."""
+    """Y - qm lies in [-m, m), and entry m + (Y - qm) of the rotated table
+    (entry i: the residue (i - 2^31) mod m) is Ã mod m."""
     rng = np.random.default_rng(m)
     At = residue_samples(rng)
-    b, u1, u2, u3 = limbs_of(At)
-    Y, exact = limb_sum(b, u1, u2, u3, m)
-    assert np.all((exact > 4 * (1 << 24)) & (exact < 4 * (1 << 28)))   # 2^24 < y < 2^28
+    Y, exact = limb_sum(*limbs_of(At), m)
+    assert np.all((exact > 0) & (exact < 1 << 32))
     assert np.array_equal(Y.astype(np.int64), exact)
-    magic = -(-(1 << 30) // m)
+    magic = -(-(1 << 32) // m)
+    assert magic < 1 << 32
     q = mulhi(Y, magic).astype(np.int64)
-    off = exact - q * 4 * m
-    assert np.all((off >= -4 * m) & (off < 4 * m) & (off % 4 == 0))
-    entry = m + off // 4
+    off = exact - q * m
+    assert np.all((off >= -m) & (off < m))
+    entry = m + off
     assert np.array_equal(np.mod(entry - BIAS, m), np.mod(At, m))
+
+
+@pytest.mark.parametrize("m", [m for m in orc.moduli(16) if not orc.square_base(m)] + [1089, 529])
+def test_limb_sum_stays_in_range_at_the_extremes(m):
+    """The sum's bounds at the limbs' extreme values: v0 ∈ [0, 2^21),
+    v1 ∈ [0, 2^21), v2 ∈ [-2^20, 2^20), with the square moduli's added
+    constant below m."""
+    c1, c2 = centred_weight(1, m), centred_weight(2, m)
+    lo = BIAS + min(0, c1) * ((1 << LIMB) - 1) + min(-c2 * (1 << 20), c2 * ((1 << 20) - 1))
+    hi = BIAS + (1 << LIMB) - 1 + m + max(0, c1) * ((1 << LIMB) - 1) + max(-c2 * (1 << 20), c2 * ((1 << 20) - 1))
+    assert 0 < lo and hi < 1 << 32
 
 
 @pytest.mark.parametrize("m", [m for m in orc.moduli(16) if orc.square_base(m)])
@@ -158,14 +178,14 @@ def test_square_digits(m):
     assert shift >= 0
     rng = np.random.default_rng(m)
     At = residue_samples(rng)
-    b, u1, u2, u3 = limbs_of(At)
-    Y, exact = limb_sum(b, u1, u2, u3, m, extra=E)
-    assert np.all((exact > 4 * (1 << 24)) & (exact < 4 * (1 << 28)))   # 2^24 < y < 2^28
+    Y, exact = limb_sum(*limbs_of(At), m, extra=E)
+    assert np.all((exact > 0) & (exact < 1 << 32))
     assert np.array_equal(Y.astype(np.int64), exact)
-    q = mulhi(Y, -(-(1 << 30) // m)).astype(np.int64)
-    off = exact - q * 4 * m
-    off = np.where(off < 0, off + 4 * m, off)
-    u = (off >> 2) + shift
+    q = mulhi(Y, -(-(1 << 32) // m)).astype(np.int64)
+    off = exact - q * m
+    assert np.all((off >= -m) & (off < m))
+    off = np.where(off < 0, off + m, off)
+    u = off + shift
     a1 = u >> 5 if s == 32 else mulhi(u, -(-(1 << 32) // s)).astype(np.int64)
     a0 = u - a1 * s
     d0, d1 = orc.square_digits(orc.centred(At, m), s)
