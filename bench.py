@@ -45,17 +45,23 @@ FP8_TO_BF16 = 2.0   # nominal dense FP8 / BF16 tensor ratio (4.5 / 2.25 PFLOP/s)
 NOMINAL_FP8_TFLOPS = 4500.0  # nominal dense FP8 tensor rate of one GB300
 PAPER_FP8_TFLOPS = 5000.0    # the paper's B300/GB300 dense FP8 figure (its Table of specs)
 PAPER_HBM_GBS = 8000.0       # the paper's B300/GB300 HBM figure
-GEMM_SOURCE = os.path.join(ROOT, "paper_2606_06510_gb300", "csrc", "k_gemm.cu")
+# The residue GEMM's sources: the kernel and the device headers it compiles.
+GEMM_SOURCES = [os.path.join(ROOT, "paper_2606_06510_gb300", "csrc", f)
+                for f in ("k_gemm.cu", "oz2_gemm.cuh", "oz2_common.cuh")]
 # DRAM read+write bytes of one residue-GEMM launch at 4096^3, r = 12, from
-# one ncu capture of that launch; reported only while the kernel source is
-# the one the counters were taken on.
+# one ncu capture of that launch; reported only while the kernel's sources
+# are the ones the counters were taken on (SHA-256 over them in order).
 GEMM_TRAFFIC = {"workload": "dgemm_4096", "num_moduli": 12, "bytes": 2.1354e9,
                 "sha256": "b789d94bee8d2079280d7c8cdd1877cb43be95b7cbed656bdf6d6998779cdae1"}
 
 
 def gemm_traffic(w, r):
     try:
-        sha = hashlib.sha256(open(GEMM_SOURCE, "rb").read()).hexdigest()
+        h = hashlib.sha256()
+        for f in GEMM_SOURCES:
+            with open(f, "rb") as fh:
+                h.update(fh.read())
+        sha = h.hexdigest()
     except OSError:
         return None
     t = GEMM_TRAFFIC
