@@ -157,13 +157,16 @@ __host__ __device__ __forceinline__ int64_t rows_stored(int64_t rows) {
   return MODE == 0 ? rows : (rows + kPlaneRows - 1) / kPlaneRows * kPlaneRows;
 }
 
-// Gather byte `b` of four 32-bit words into one word (byte 0 from w0 ...).
-__device__ __forceinline__ uint32_t gather_byte(uint32_t w0, uint32_t w1, uint32_t w2, uint32_t w3,
-                                                int b) {
-  uint32_t sel = static_cast<uint32_t>(b) | (static_cast<uint32_t>(b + 4) << 4);
-  uint32_t lo = __byte_perm(w0, w1, sel);       // bytes: w0.b, w1.b
-  uint32_t hi = __byte_perm(w2, w3, sel);       // bytes: w2.b, w3.b
-  return __byte_perm(lo, hi, 0x5410);
+// Bytes 0, 1 and 2 of four 32-bit words w0..w3 gathered into p0, p1, p2
+// (byte j of p_b is byte b of w_j): a 4 × 4 byte transpose in two rounds of
+// byte permutes, seven in all.
+__device__ __forceinline__ void transpose3(uint32_t w0, uint32_t w1, uint32_t w2, uint32_t w3, uint32_t& p0,
+                                           uint32_t& p1, uint32_t& p2) {
+  const uint32_t t0 = __byte_perm(w0, w1, 0x5140), t1 = __byte_perm(w0, w1, 0x7362);  // w0.b0 w1.b0 w0.b1 w1.b1 | .b2 .b3
+  const uint32_t t2 = __byte_perm(w2, w3, 0x5140), t3 = __byte_perm(w2, w3, 0x7362);
+  p0 = __byte_perm(t0, t2, 0x5410);
+  p1 = __byte_perm(t0, t2, 0x7632);
+  p2 = __byte_perm(t1, t3, 0x5410);
 }
 
 struct OperandView {
@@ -236,11 +239,24 @@ __device__ __forceinline__ void square_digits(const Limbs& L, uint8_t* dst) {
     const uint32_t q = __umulhi(Y, mc.magic);
     int off = static_cast<int>(Y - q * static_cast<uint32_t>(mc.m));  // (Y mod m) or that - m
     off += off < 0 ? mc.m : 0;
-    const uint32_t u = static_cast<uint32_t>(off) + kShift;
-    const uint32_t a1 = mc.s == 32 ? u >> 5 : __umulhi(u, mc.sq_magic);
-    const uint32_t a0 = u - a1 * static_cast<uint32_t>(mc.s);
-    f0[e] = small_int_float(a0 + (0x4B400000u - mc.sq_h0));
-    f1[e] = small_int_float(a1 + (0x4B400000u - mc.sq_h1));
+    if constexpr (mc.s == 32) {
+      const uint32_t u = static_cast<uint32_t>(off) + kShift;
+      f0[e] = small_int_float((u & 31u) + (0x4B400000u - mc.sq_h0));
+      f1[e] = small_int_float((u >> 5) + (0x4B400000u - mc.sq_h1));
+    } else {
+      // u = off + kShift as the float with bits 0x4B400000 + u (1.5·2^23 + u).
+      // t = RD(u·(c17/2^17) + 1.5·2^23) = 1.5·2^23 + ⌊u/s⌋ (the grid there
+      // is the integers, and u·c17/2^17 is within u/2^17 < 1/s of u/s);
+      // d1 = t - (1.5·2^23 + h1), d0 = (u - h0 - s·h1) - s·d1.  Every value
+      // is an integer below 2^24, exact in FP32, and the FP32 pipes take
+      // this work off the integer multiply pipe the residue sums load.
+      const float ub = __int_as_float(static_cast<int>(static_cast<uint32_t>(off) + (0x4B400000u + kShift)));
+      const float uf = ub - 12582912.0f;
+      const float uh = ub - static_cast<float>(12582912 + mc.sq_h0 + mc.s * mc.sq_h1);
+      const float t = __fmaf_rd(uf, static_cast<float>(mc.sq_c17) * (1.0f / 131072.0f), 12582912.0f);
+      f1[e] = t - static_cast<float>(12582912 + mc.sq_h1);
+      f0[e] = __fmaf_rn(-static_cast<float>(mc.s), f1[e], uh);
+    }
   }
   uint8_t* pdst = dst + (mc.plane_off - PBASE) * STRIDE;
   *reinterpret_cast<uint2*>(pdst) = make_uint2(__byte_perm(e4m3x2(f0[0], f0[1]), e4m3x2(f0[2], f0[3]), 0x5410),
@@ -268,10 +284,11 @@ __device__ __forceinline__ void planes_one(const Limbs& L, const uint32_t* table
     w[e] = centre[off];  // packed E4M3 planes of centred(Ã mod m)
   }
   uint8_t* pdst = dst + (mc.plane_off - PBASE) * STRIDE;
+  uint32_t lo[3], hi[3];
+  transpose3(w[0], w[1], w[2], w[3], lo[0], lo[1], lo[2]);
+  transpose3(w[4], w[5], w[6], w[7], hi[0], hi[1], hi[2]);
 #pragma unroll
-  for (int p = 0; p < (mc.s ? 2 : 3); ++p)
-    *reinterpret_cast<uint2*>(pdst + p * STRIDE) =
-        make_uint2(gather_byte(w[0], w[1], w[2], w[3], p), gather_byte(w[4], w[5], w[6], w[7], p));
+  for (int p = 0; p < 3; ++p) *reinterpret_cast<uint2*>(pdst + p * STRIDE) = make_uint2(lo[p], hi[p]);
 }
 
 template <int... Is>

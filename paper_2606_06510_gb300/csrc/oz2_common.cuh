@@ -53,10 +53,10 @@ struct ModConst {
   uint32_t magic; // ⌈2^32/m⌉
   // Square moduli (digits computed, not looked up): E = (⌊m/2⌋ - kDecBias)
   // mod m, the digit offsets h0 = ⌊s/2⌋ and h1 = ⌈(⌊m/2⌋ - h0)/s⌉, and
-  // ⌈2^32/s⌉.
+  // ⌈2^17/s⌉ (⌊u·⌈2^17/s⌉/2^17⌋ = ⌊u/s⌋ for u < 2^17/s).
   uint32_t sq_e;
   int sq_h0, sq_h1;
-  uint32_t sq_magic;
+  int sq_c17;
 };
 
 // x mod m in [-⌊m/2⌋, m - 1 - ⌊m/2⌋] (the centred residue) for x ≥ 0.
@@ -111,7 +111,7 @@ constexpr ModConst mod_const(int i) {
     c.sq_e = static_cast<uint32_t>((static_cast<long long>(H) - kDecBias % um + m) % m);
     c.sq_h0 = c.s / 2;
     c.sq_h1 = (H - c.sq_h0 + c.s - 1) / c.s;
-    c.sq_magic = static_cast<uint32_t>(((1ull << 32) + c.s - 1) / static_cast<unsigned long long>(c.s));
+    c.sq_c17 = ((1 << 17) + c.s - 1) / c.s;
   }
   return c;
 }
@@ -151,13 +151,13 @@ struct Oz2Moduli {
   int crt_g[kMaxModuli];
   int crt_ml, crt_mlh;
   int crt_m51l, crt_m51h;
-  // 96-bit direct CRT (r = 11, 12): F_k = round(2^96·y_k/m_k) = y2·2^64 + y1·2^32 + y0
-  // with y0 and y1 signed low words; M as four 32-bit words; and bounds on
-  // |X| - ⌊|Y|·M/2^96⌋ for centred residues and for any int16 residues.
+  // 96-bit direct CRT of the fused kernel (r = 11, 12): F_k = round(2^96·y_k/m_k)
+  // = y2·2^64 + y1·2^32 + y0 with y0 and y1 signed low words; M as four
+  // 32-bit words; and a bound on |X| - ⌊|Y|·M/2^96⌋ for centred residues.
   int crt_y0[kMaxModuli], crt_y1[kMaxModuli];
   uint32_t crt_y2[kMaxModuli];
   uint32_t crt_m32[4];
-  unsigned long long crt_err_centred, crt_err_any;
+  unsigned long long crt_err_centred;
   int table_entries;            // 2·Σ m_i over the nonsquare moduli (digit-plane table)
 };
 
@@ -455,6 +455,31 @@ __host__ __device__ constexpr uint32_t idesc_f8_f32(int M, int N) {
 namespace oz2 {
 // Counts kernel launches made by the library (read through oz2_get_stats).
 void count_launch(int n = 1);
+
+// Programmatic dependent launch: the kernel may be scheduled while the
+// kernel before it in the stream is still running (once every block of that
+// one has called pdl_trigger() or exited), so its launch latency overlaps
+// the predecessor's tail.  It must call pdl_wait(), which returns once the
+// predecessor has completed and its writes are visible, before it reads
+// anything the predecessor wrote.  Launched the ordinary way, pdl_wait()
+// returns at once.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_dependent(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                                   Args... args) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 struct ScanOut {
   int32_t* ra;
   int32_t* cb;
@@ -496,7 +521,7 @@ cudaError_t launch_plane_gemm(int64_t m, int64_t n, int64_t k_pad, const Oz2Modu
 // GEMM writes them); otherwise any int16 representative.
 cudaError_t launch_reconstruct(int64_t m, int64_t n, const Oz2Moduli& mods,
                                const int16_t* residues, int64_t ldr, const int32_t* d,
-                               const int32_t* e, double* C, int64_t ldc, bool centred, cudaStream_t st);
+                               const int32_t* e, double* C, int64_t ldc, cudaStream_t st);
 cudaError_t launch_fallback_lists(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda,
                                   const double* B, int64_t ldb, const uint8_t* row_flag,
                                   const uint8_t* col_flag, int* scratch, double* C, int64_t ldc,

@@ -165,10 +165,25 @@ def test_limb_sum_stays_in_range_at_the_extremes(m):
     assert 0 < lo and hi < 1 << 32
 
 
+def square_digits_fp(u, s, h0, h1):
+    """The kernel's FP32 digits of u = c + h0 + s·h1 for s ≠ 32: the float
+    1.5·2^23 + u, one fused multiply-add rounded down,
+    t = 1.5·2^23 + ⌊u·⌈2^17/s⌉/2^17⌋ (exact: the grid at 1.5·2^23 is the
+    integers), d1 = t - (1.5·2^23 + h1), d0 = (u - h0 - s·h1) - s·d1."""
+    c17 = -(-(1 << 17) // s)
+    base = 3 << 22
+    t = base + (u * c17) // (1 << 17)
+    d1 = t - (base + h1)
+    d0 = (u - h0 - s * h1) - s * d1
+    return d0, d1, t
+
+
 @pytest.mark.parametrize("m", [m for m in orc.moduli(16) if orc.square_base(m)])
 def test_square_digits(m):
-    """The computed balanced base-s digits equal the oracle's digits of the
-    centred residue."""
+    """The kernel's square digits from the limbs of Ã equal the oracle's
+    digits of the centred residue: the sum with the added constant, the
+    corrected remainder, then a shift and mask for s = 32 and the FP32
+    form for the other bases."""
     s = orc.square_base(m)
     H = m // 2
     E = (H - BIAS) % m
@@ -186,7 +201,29 @@ def test_square_digits(m):
     assert np.all((off >= -m) & (off < m))
     off = np.where(off < 0, off + m, off)
     u = off + shift
-    a1 = u >> 5 if s == 32 else mulhi(u, -(-(1 << 32) // s)).astype(np.int64)
-    a0 = u - a1 * s
-    d0, d1 = orc.square_digits(orc.centred(At, m), s)
-    assert np.array_equal(a0 - h0, d0) and np.array_equal(a1 - h1, d1)
+    if s == 32:
+        d0, d1 = (u & 31) - h0, (u >> 5) - h1
+    else:
+        d0, d1, _ = square_digits_fp(u, s, h0, h1)
+    w0, w1 = orc.square_digits(orc.centred(At, m), s)
+    assert np.array_equal(d0, w0) and np.array_equal(d1, w1)
+
+
+@pytest.mark.parametrize("m", [m for m in orc.moduli(16) if orc.square_base(m) and orc.square_base(m) != 32])
+def test_square_digits_by_fp32_fma(m):
+    """The FP32 form of the square digits over every centred residue: the
+    rounded-down fused multiply-add gives ⌊u/s⌋ exactly, the digits match
+    the oracle's, and every operand and result is an integer below 2^24."""
+    s = orc.square_base(m)
+    H = m // 2
+    h0 = s // 2
+    h1 = -(-(H - h0) // s)
+    cs = np.arange(-H, m - H)
+    u = cs + h0 + s * h1
+    base = 3 << 22
+    assert u.min() >= 0 and (base + u).max() < 1 << 24
+    d0, d1, t = square_digits_fp(u, s, h0, h1)
+    assert np.array_equal(t - base, u // s)
+    w0, w1 = orc.square_digits(cs, s)
+    assert np.array_equal(d0, w0) and np.array_equal(d1, w1)
+    assert np.abs(d0).max() <= 16 and np.abs(d1).max() <= 16
