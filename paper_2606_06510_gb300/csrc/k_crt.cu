@@ -3,13 +3,11 @@
 // and one correctly rounded (round-to-nearest-even) conversion of
 // X·2^-(d_i+e_j) to FP64, including the subnormal range.
 //
-// X is computed by the direct CRT sum in fixed point (multiply-adds only).
-// For r = 11 and 12 one 96-bit sum estimates X to about 2^28 and decides the
-// rounding whenever no midpoint between doubles lies that close; the other
-// outputs, and every output at other r, take an exact two-word or five-limb
-// direct CRT, and Garner's algorithm, the paper's method, takes over in the
-// rare case where that sum's quotient is ambiguous.  Every output equals
-// the Garner result exactly.
+// X is computed by the direct CRT sum in fixed point (multiply-adds only):
+// an exact two-word sum for r ≤ 12 and a five-limb one for r ≥ 13, with
+// Garner's algorithm, the paper's method, taking over in the rare case where
+// that sum's quotient is ambiguous.  Every output equals the Garner result
+// exactly.
 //
 // Residues arrive column-major (r matrices of m×n, ld = ldr ≥ m) from the
 // residue GEMM and C is column-major, so a thread takes two consecutive
@@ -46,9 +44,8 @@ constexpr int crt_min_blocks() {
 // (0 or 1), the first kCrtFailSlots of them; returns how many there were.
 template <int R, bool FAST>
 __device__ __forceinline__ int crt_columns(int64_t n, int64_t row, bool pair, int d0, int d1, const Oz2Moduli& mods,
-                                           unsigned long long err, const int16_t* __restrict__ res, int64_t ldr,
-                                           const int* __restrict__ e, double* cbase, int64_t ldc,
-                                           int (&fails)[kCrtFailSlots]) {
+                                           const int16_t* __restrict__ res, int64_t ldr, const int* __restrict__ e,
+                                           double* cbase, int64_t ldc, int (&fails)[kCrtFailSlots]) {
   const int64_t step = gridDim.y;
   const int64_t off_step = step * ldr;
   // Residue matrix k starts at res + k·mstride (the same for every thread,
@@ -80,7 +77,7 @@ __device__ __forceinline__ int crt_columns(int64_t n, int64_t row, bool pair, in
       for (int k = 0; k < R; ++k)
         c[k] = u ? (static_cast<int>(w[k]) >> 16) : static_cast<int>(static_cast<int16_t>(w[k] & 0xFFFFu));
       double val;
-      if (!crt_fast<R>(c, -((u ? d1 : d0) + ec), mods, err, val)) {
+      if (!crt_fast<R>(c, -((u ? d1 : d0) + ec), mods, val)) {
         val = __longlong_as_double(kCrtSentinel);
         if (nfail < kCrtFailSlots) fails[nfail] = 2 * iter + u;
         ++nfail;
@@ -130,8 +127,8 @@ __device__ __forceinline__ int crt_columns(int64_t n, int64_t row, bool pair, in
 template <int R, bool FAST>
 __global__ void __launch_bounds__(kCrtThreads, crt_min_blocks<R, FAST>())
     crt_kernel(int64_t row0, int64_t rows, int64_t n, const __grid_constant__ Oz2Moduli mods,
-               unsigned long long err, const int16_t* __restrict__ res, int64_t ldr, const int* __restrict__ d,
-               const int* __restrict__ e, double* __restrict__ C, int64_t ldc) {
+               const int16_t* __restrict__ res, int64_t ldr, const int* __restrict__ d, const int* __restrict__ e,
+               double* __restrict__ C, int64_t ldc) {
   const int64_t rel = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) * 2;
   if (rel >= rows) return;
   const int64_t row = row0 + rel;
@@ -139,7 +136,7 @@ __global__ void __launch_bounds__(kCrtThreads, crt_min_blocks<R, FAST>())
   const int d0 = d[row], d1 = pair ? d[row + 1] : 0;
   double* cbase = C + row;
   int fails[kCrtFailSlots];
-  const int nfail = crt_columns<R, FAST>(n, row, pair, d0, d1, mods, err, res, ldr, e, cbase, ldc, fails);
+  const int nfail = crt_columns<R, FAST>(n, row, pair, d0, d1, mods, res, ldr, e, cbase, ldc, fails);
   if (nfail == 0) return;
   // Outputs the fast path left to the exact paths (this thread's own).
   const int64_t step = gridDim.y;
@@ -164,8 +161,8 @@ __global__ void __launch_bounds__(kCrtThreads, crt_min_blocks<R, FAST>())
 // over the columns, about two waves of resident blocks in all.
 template <int R, bool FAST>
 static cudaError_t launch_crt_rows(cudaStream_t st, int64_t row0, int64_t rows, int64_t n, const Oz2Moduli& mods,
-                                   unsigned long long err, const int16_t* res, int64_t ldr, const int32_t* d,
-                                   const int32_t* e, double* C, int64_t ldc) {
+                                   const int16_t* res, int64_t ldr, const int32_t* d, const int32_t* e, double* C,
+                                   int64_t ldc) {
   int dev = 0, sms = 148;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
@@ -177,34 +174,32 @@ static cudaError_t launch_crt_rows(cudaStream_t st, int64_t row0, int64_t rows, 
   gy = gy > 65535 ? 65535 : gy;
   count_launch();
   crt_kernel<R, FAST><<<dim3(static_cast<unsigned>(gx), static_cast<unsigned>(gy)), kCrtThreads, 0, st>>>(
-      row0, rows, n, mods, err, res, ldr, d, e, C, ldc);
+      row0, rows, n, mods, res, ldr, d, e, C, ldc);
   return cudaGetLastError();
 }
 
 template <int R>
-static cudaError_t launch_crt_r(cudaStream_t st, int64_t m, int64_t n, const Oz2Moduli& mods,
-                                unsigned long long e96, const int16_t* res, int64_t ldr, const int32_t* d,
-                                const int32_t* e, double* C, int64_t ldc) {
+static cudaError_t launch_crt_r(cudaStream_t st, int64_t m, int64_t n, const Oz2Moduli& mods, const int16_t* res,
+                                int64_t ldr, const int32_t* d, const int32_t* e, double* C, int64_t ldc) {
   const bool vec = (ldr % 2 == 0) && (reinterpret_cast<uintptr_t>(res) % 4 == 0) && (ldc % 2 == 0) &&
                    (reinterpret_cast<uintptr_t>(C) % 16 == 0);
-  if (!vec) return launch_crt_rows<R, false>(st, 0, m, n, mods, e96, res, ldr, d, e, C, ldc);
+  if (!vec) return launch_crt_rows<R, false>(st, 0, m, n, mods, res, ldr, d, e, C, ldc);
   const int64_t even = m & ~int64_t{1};
   cudaError_t err = cudaSuccess;
-  if (even > 0) err = launch_crt_rows<R, true>(st, 0, even, n, mods, e96, res, ldr, d, e, C, ldc);
+  if (even > 0) err = launch_crt_rows<R, true>(st, 0, even, n, mods, res, ldr, d, e, C, ldc);
   if (err == cudaSuccess && even < m)
-    err = launch_crt_rows<R, false>(st, even, 1, n, mods, e96, res, ldr, d, e, C, ldc);
+    err = launch_crt_rows<R, false>(st, even, 1, n, mods, res, ldr, d, e, C, ldc);
   return err;
 }
 
 cudaError_t launch_reconstruct(int64_t m, int64_t n, const Oz2Moduli& mods, const int16_t* residues,
                                int64_t ldr, const int32_t* d, const int32_t* e, double* C, int64_t ldc,
-                               bool centred, cudaStream_t st) {
+                               cudaStream_t st) {
   if (m == 0 || n == 0) return cudaSuccess;
-  const unsigned long long e96 = centred ? mods.crt_err_centred : mods.crt_err_any;
   switch (mods.r) {
 #define OZ2_CRT_CASE(R) \
   case R:               \
-    return launch_crt_r<R>(st, m, n, mods, e96, residues, ldr, d, e, C, ldc);
+    return launch_crt_r<R>(st, m, n, mods, residues, ldr, d, e, C, ldc);
     OZ2_CRT_CASE(1) OZ2_CRT_CASE(2) OZ2_CRT_CASE(3) OZ2_CRT_CASE(4) OZ2_CRT_CASE(5) OZ2_CRT_CASE(6)
     OZ2_CRT_CASE(7) OZ2_CRT_CASE(8) OZ2_CRT_CASE(9) OZ2_CRT_CASE(10) OZ2_CRT_CASE(11) OZ2_CRT_CASE(12)
     OZ2_CRT_CASE(13) OZ2_CRT_CASE(14) OZ2_CRT_CASE(15) OZ2_CRT_CASE(16)

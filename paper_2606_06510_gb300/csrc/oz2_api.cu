@@ -188,11 +188,11 @@ static Oz2Moduli build_moduli(int r, int quant) {
   u64 M[3] = {1, 0, 0};
   for (int i = 0; i < r; ++i) mul3(M, static_cast<u64>(kModuliAll[i]));
   for (int i = 0; i < 3; ++i) c.M[i] = M[i];
-  // 96-bit constants (used for r ≤ 12, M < 2^112): F_k = round(2^96·y_k/m_k)
-  // split into signed low words, and the error bound of the estimate of |X|:
-  // |X| - ⌊|Y|·M/2^96⌋ (partial products below 2^64 dropped) is within
-  // (Σ_k cmax_k)·M/2^97 + 5 < (Σ cmax_k)·(⌊M/2^64⌋ + 1)/2^33 + 5, with cmax_k
-  // = ⌊m_k/2⌋ for centred residues and 2^15 for any int16 residue.
+  // 96-bit constants (the fused kernel, r = 11, 12, M < 2^112): F_k =
+  // round(2^96·y_k/m_k) split into signed low words, and the error bound of
+  // the estimate of |X|: |X| - ⌊|Y|·M/2^96⌋ (partial products below 2^64
+  // dropped) is within (Σ_k ⌊m_k/2⌋)·M/2^97 + 5 <
+  // (Σ ⌊m_k/2⌋)·(⌊M/2^64⌋ + 1)/2^33 + 5 for centred residues.
   {
     u64 sum_centred = 0;
     for (int k = 0; k < r; ++k) {
@@ -213,9 +213,7 @@ static Oz2Moduli build_moduli(int r, int quant) {
     }
     for (int i = 0; i < 4; ++i) c.crt_m32[i] = static_cast<uint32_t>(M[i >> 1] >> (32 * (i & 1)));
     const unsigned __int128 mh1 = static_cast<unsigned __int128>(M[1]) + 1;  // M < 2^128 here
-    const u64 sum_any = 32768ull * static_cast<u64>(r);
     c.crt_err_centred = static_cast<u64>((sum_centred * mh1 + ((static_cast<unsigned __int128>(1) << 33) - 1)) >> 33) + 6;
-    c.crt_err_any = static_cast<u64>((sum_any * mh1 + ((static_cast<unsigned __int128>(1) << 33) - 1)) >> 33) + 6;
   }
   split_signed_low(M[0], &c.crt_ml, &c.crt_mlh);
   // round(M/2^51), below 2^61 while M < 2^112 (r ≤ 12, the only use).
@@ -622,7 +620,7 @@ static int run_stages(int64_t m, int64_t n, int64_t k, const double* A, int64_t 
       }
       mark(6);
       if (err == cudaSuccess)
-        err = launch_reconstruct(m, cols, mods, res, L.res_ld, d, e + c0, C + c0 * ldc, ldc, true, s);
+        err = launch_reconstruct(m, cols, mods, res, L.res_ld, d, e + c0, C + c0 * ldc, ldc, s);
       mark(7);
     }
     if (err == cudaSuccess)
@@ -986,7 +984,7 @@ int oz2_reconstruct(int64_t m, int64_t n, int num_moduli, const int16_t* residue
   if (m && n && (!residues || !d || !e || !C)) return OZ2_ERR_INVALID_ARG;
   const Oz2Moduli mods = build_moduli(num_moduli, OZ2_QUANT_TZ);
   return to_status(
-      launch_reconstruct(m, n, mods, residues, ldr, d, e, C, ldc, false, static_cast<cudaStream_t>(stream)));
+      launch_reconstruct(m, n, mods, residues, ldr, d, e, C, ldc, static_cast<cudaStream_t>(stream)));
 }
 
 int oz2_fallback(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, const double* B, int64_t ldb,

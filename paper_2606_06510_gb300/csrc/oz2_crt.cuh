@@ -296,7 +296,7 @@ __device__ __forceinline__ bool crt_value_w64(const int (&c)[R], int E, const Oz
   return true;
 }
 
-// Fast path for r = 11, 12 (2^102 < M < 2^112): one 96-bit fixed-point sum.
+// 96-bit estimate for r = 11, 12 (2^102 < M < 2^112): one fixed-point sum.
 // With F_k = round(2^96·y_k/m_k), Y = Σ c_k F_k mod 2^96 read as a signed
 // word is 2^96·X/M + D with |D| ≤ Σ|c_k|/2, as long as that stays inside
 // [-2^95, 2^95) (|Y| < 2^95 - 2^64 shows there was no wrap).  Then
@@ -372,37 +372,18 @@ __device__ __forceinline__ bool y96_finish(const Y96& y, int E, const Oz2Moduli&
   return true;
 }
 
-template <int R>
-__device__ __forceinline__ bool crt_value_y96(const int (&c)[R], int E, const Oz2Moduli& mods,
-                                              unsigned long long err, double& out) {
-  Y96 y{0, 0, 0u};
-#pragma unroll
-  for (int k = 0; k < R; ++k) y96_add(y, c[k], mods, k);
-  if ((y.a0 | y.a1 | static_cast<long long>(y.a2)) == 0) {
-    // Y = 0: X is 0 when every residue is (rows and columns that are zero in
-    // the emulation), whose result is +0; any other X takes the exact path.
-    int any = 0;
-#pragma unroll
-    for (int k = 0; k < R; ++k) any |= c[k];
-    out = 0.0;
-    return any == 0;
-  }
-  return y96_finish(y, E, mods, err, out);
-}
-
 constexpr long long kCrtSentinel = 0x7FF4DEAD0BADF00Dll;  // a NaN the reconstruction never produces
 
-// The fast path by moduli count: the 96-bit estimate for r = 11, 12 (M of
-// 103 and 112 bits: |X| is then above 2^85 except in rare outputs); the
-// exact two-word CRT for r ≤ 10, where X has at most 94 bits and an
-// estimate within ±err decides fewer roundings; the five-limb CRT for
-// r ≥ 13.
+// The reconstruction kernel's fast path by moduli count: the exact two-word
+// direct CRT for r ≤ 12 (it defers only when X lies within M/2^12 of ±M/2)
+// and the five-limb one for r ≥ 13.  (The 96-bit estimate above costs fewer
+// multiplies but defers small and near-midpoint outputs; measured on one
+// GB300 it was 3% slower at 4096³ and, on wide-range data with many small
+// outputs, 20% slower, so only the fused kernel, whose per-output state must
+// stay small, uses it.)
 template <int R>
-__device__ __forceinline__ bool crt_fast(const int (&c)[R], int E, const Oz2Moduli& mods, unsigned long long err,
-                                         double& out) {
-  if constexpr (R >= 11 && R <= 12)
-    return crt_value_y96<R>(c, E, mods, err, out);
-  else if constexpr (R <= 10)
+__device__ __forceinline__ bool crt_fast(const int (&c)[R], int E, const Oz2Moduli& mods, double& out) {
+  if constexpr (R <= 12)
     return crt_value_w64<R>(c, E, mods, out);
   else
     return crt_value_fast<R>(c, E, mods, out);

@@ -1,6 +1,7 @@
-"""The reconstruction's 96-bit fast path (r = 11, 12), on the CPU.
+"""The fused kernel's 96-bit CRT estimate (r = 11, 12), on the CPU.
 
-The CUDA reconstruction estimates X from one fixed-point sum: with
+The fused residue-GEMM + reconstruction kernel folds each modulus's residue
+into one fixed-point sum per output and estimates X from it: with
 F_k = round(2^96·y_k/m_k), Y = Σ c_k F_k mod 2^96 (a signed word) is
 2^96·X/M + D with |D| ≤ Σ|c_k|/2, and P = ⌊|Y|·M/2^96⌋ (partial products of
 32-bit words below 2^64 dropped) is within a host-computed bound err of |X|.
@@ -9,8 +10,9 @@ within err of P; otherwise an exact path runs.  These tests build the
 constants here from their definitions, check the bound against the worst
 residues, emulate the word arithmetic on Python integers, and compare every
 value the fast path returns with the correctly rounded X·2^E (float of an
-exact rational), including X placed next to midpoints and non-centred
-residue representatives.
+exact rational), including X placed next to midpoints.  The kernel sees
+centred residues; the cases with other representatives check the same
+arithmetic under the wider bound those need.
 """
 from fractions import Fraction
 import math
@@ -63,8 +65,6 @@ def fast_path(c, E, r, err):
     a1 = sum(ck * f1 for ck, (_, _, _, _, f1, _) in zip(c, ks))
     a2 = sum(ck * f2 for ck, (_, _, _, _, _, f2) in zip(c, ks)) & MASK32
     assert -2 ** 63 <= a0 < 2 ** 63 and -2 ** 63 <= a1 < 2 ** 63
-    if a0 == 0 and a1 == 0 and a2 == 0:      # Y = 0: X = 0 when every residue is
-        return 0.0 if not any(c) else None
     s1 = (a0 >> 32) + a1
     w0, w1 = a0 & MASK32, s1 & MASK32
     w2 = ((s1 >> 32) + a2) & MASK32
@@ -188,8 +188,7 @@ def test_small_and_subnormal_results_defer():
     r = 12
     M, mods, _ = constants(r)
     err = err_bound(M, mods, True)
-    assert fast_path(residues(0, mods), -10, r, err) == 0.0      # all residues zero: +0
-    for x in (5, -(2 ** 40), 2 ** 80):
+    for x in (0, 5, -(2 ** 40), 2 ** 80):
         assert fast_path(residues(x, mods), -10, r, err) is None
     x = 2 ** 100 + 12345
     assert fast_path(residues(x, mods), -1200, r, err) is None      # subnormal result

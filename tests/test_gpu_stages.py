@@ -254,10 +254,10 @@ def test_reconstruct_tiles_and_alignment(oz, r, m, n, ldr, ldc, c_off):
 
 def test_reconstruct_many_outputs_left_to_the_exact_path(oz):
     """Two rows and more columns than the launch has column strides, so each
-    thread walks about ten columns, with most outputs small (|X| < 2^80),
-    which the 96-bit fast path of r = 12 leaves to the exact path: threads
-    leave more outputs than their list holds and find the rest again by
-    rescanning; large, zero and midpoint-free outputs are mixed in."""
+    thread walks about ten columns, with most outputs within M/2^13 of ±M/2,
+    which the fast path leaves to Garner's algorithm: threads leave more
+    outputs than their list holds and find the rest again by rescanning;
+    small, zero and other outputs are mixed in."""
     import random
     import torch
     r = 12
@@ -266,12 +266,17 @@ def test_reconstruct_many_outputs_left_to_the_exact_path(oz):
     rng = random.Random(77)
     m, n = 2, 12500
     xs = []
+    lo, hi, band = -(M // 2), M - M // 2 - 1, M >> 13
     for _ in range(m * n):
         t = rng.random()
-        if t < 0.7:
-            xs.append(rng.randrange(-(1 << 80), 1 << 80))
+        if t < 0.35:
+            xs.append(lo + rng.randrange(band))
+        elif t < 0.7:
+            xs.append(hi - rng.randrange(band))
         elif t < 0.8:
             xs.append(0)
+        elif t < 0.9:
+            xs.append(rng.randrange(-(1 << 80), 1 << 80))
         else:
             xs.append(rng.randrange(-(M // 4), M // 4))
     X = np.array(xs, dtype=object).reshape(m, n)
