@@ -212,7 +212,10 @@ int oz2_workspace_layout(int64_t m, int64_t n, int64_t k, int num_moduli,
 
 /* How the library runs a problem on a GPU with cta_pairs CTA pairs (half its
  * SM count: 76 on a GB300).  Host arithmetic only: it touches no device and
- * runs without one.
+ * runs without one.  A call on a device uses min(SMs/2, the residue GEMM's
+ * resident two-CTA clusters) pairs, which is SMs/2 unless another kernel's
+ * resources or a partitioned device cut the resident clusters; the plan
+ * matches a call only for the pair count that call used.
  *   kparts        parts of k per residue-GEMM unit in oz2_dgemm_ex and
  *                 oz2_dgemm (1: no split).  A small C with a long k fills
  *                 few waves of the CTA pairs; each unit then covers 1/kparts

@@ -90,6 +90,7 @@ struct ScanGrid {
 __global__ void __launch_bounds__(256) scan_kernel(int64_t m, int64_t n, int64_t k, const double* __restrict__ A,
                                                    int64_t lda, const double* __restrict__ B, int64_t ldb, ScanGrid g,
                                                    int* __restrict__ ra, int* __restrict__ cb) {
+  pdl_trigger();  // the flags kernel may be scheduled now; it waits for this grid to finish
   const int64_t b = blockIdx.x;
   if (b < g.ga) {
     scan_a_rows(b % g.gax, b / g.gax, m, k, A, lda, g.achunk, ra);
@@ -116,6 +117,7 @@ __global__ void __launch_bounds__(kFinalizeThreads) finalize_flags_kernel(int64_
   __shared__ int warp_sum[32];
   __shared__ int med_s;
   __shared__ int count_s;
+  pdl_wait();  // the scan keys are complete
   const bool is_a = blockIdx.x == 0;
   const int64_t cnt = is_a ? m : n;
   int* key = is_a ? ra : cb;
@@ -227,9 +229,9 @@ cudaError_t launch_scan(int64_t m, int64_t n, int64_t k, const double* A, int64_
     scan_kernel<<<static_cast<unsigned>(g.ga + gb), 256, 0, st>>>(m, n, k, A, lda, B, ldb, g, out.ra, out.cb);
   }
   count_launch();
-  finalize_flags_kernel<<<2, kFinalizeThreads, 0, st>>>(m, n, out.ra, out.cb, out.row_flag, out.col_flag,
-                                            flags, dev);
-  return cudaGetLastError();
+  const cudaError_t e2 = launch_dependent(finalize_flags_kernel, dim3(2), dim3(kFinalizeThreads), 0, st, m, n, out.ra,
+                                          out.cb, out.row_flag, out.col_flag, flags, dev);
+  return e2 != cudaSuccess ? e2 : cudaGetLastError();
 }
 
 // ---------------------------------------------------------------------------
