@@ -348,6 +348,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           tmem_ld16(lane_addr + c, v0);
           if (MODE == 0) tmem_ld16(lane_addr + kAccCols + c, v1);
           tmem_ld_wait();
+          if (c == 48 && !carry) {
+            // The last chunk is in registers: release the accumulators now,
+            // so the next unit's MMAs overlap this chunk's reduction and
+            // stores.
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive_remote(acc_empty_leader);
+          }
           if (MODE == 1) {
 #pragma unroll
             for (int j = 0; j < 16; ++j) rowmax = fmaxf(rowmax, __uint_as_float(v0[j]));
@@ -407,10 +415,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
             }
           }
         }
-        if (carry) tmem_st_wait();
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive_remote(acc_empty_leader);
+        if (carry) {  // the written-back residues are in place before the next slab's MMAs
+          tmem_st_wait();
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive_remote(acc_empty_leader);
+        }
         accph ^= 1;
       }
       if (MODE == 1 && ok) {
@@ -614,7 +624,11 @@ __global__ void __launch_bounds__(kFoldThreads) fold_parts_kernel(const int16_t*
   }
 }
 
-constexpr int64_t kMaxKParts = 16;     // keeps kparts·⌊m/2⌋ < 2^16 for the fold
+// At most 16 parts of k.  The fold's sum of kparts centred residues stays
+// far inside 16 bits (16·⌊m/2⌋ ≤ 8704); what limits a split in practice is
+// the scratch (the magnitude-plane region must hold kparts partial residue
+// sets) and the cost model's 5% gain rule.
+constexpr int64_t kMaxKParts = 16;
 constexpr int64_t kMinPartSteps = 4;   // k-blocks (512 k-entries) per part at least
 
 // Estimated duration of the residue GEMM under the unit schedule (nonsquare
