@@ -244,16 +244,18 @@ __device__ __forceinline__ void square_digits(const Limbs& L, uint8_t* dst) {
       f0[e] = small_int_float((u & 31u) + (0x4B400000u - mc.sq_h0));
       f1[e] = small_int_float((u >> 5) + (0x4B400000u - mc.sq_h1));
     } else {
-      // u = off + kShift as the float with bits 0x4B400000 + u (1.5·2^23 + u).
-      // t = RD(u·(c17/2^17) + 1.5·2^23) = 1.5·2^23 + ⌊u/s⌋ (the grid there
-      // is the integers, and u·c17/2^17 is within u/2^17 < 1/s of u/s);
+      // u = off + kShift as the float ub with bits 0x4B400000 + u
+      // (1.5·2^23 + u).  t = RD(ub·cs + (1.5·2^23 - 1.5·2^23·cs)), with
+      // cs = c17/2^17 and both terms exact (1.5·2^23·cs = 96·c17), is
+      // RD(u·cs + 1.5·2^23) = 1.5·2^23 + ⌊u/s⌋ (the grid there is the
+      // integers, and u·c17/2^17 is within u/2^17 < 1/s of u/s);
       // d1 = t - (1.5·2^23 + h1), d0 = (u - h0 - s·h1) - s·d1.  Every value
       // is an integer below 2^24, exact in FP32, and the FP32 pipes take
       // this work off the integer multiply pipe the residue sums load.
       const float ub = __int_as_float(static_cast<int>(static_cast<uint32_t>(off) + (0x4B400000u + kShift)));
-      const float uf = ub - 12582912.0f;
       const float uh = ub - static_cast<float>(12582912 + mc.sq_h0 + mc.s * mc.sq_h1);
-      const float t = __fmaf_rd(uf, static_cast<float>(mc.sq_c17) * (1.0f / 131072.0f), 12582912.0f);
+      const float t = __fmaf_rd(ub, static_cast<float>(mc.sq_c17) * (1.0f / 131072.0f),
+                                static_cast<float>(12582912 - 96 * mc.sq_c17));
       f1[e] = t - static_cast<float>(12582912 + mc.sq_h1);
       f0[e] = __fmaf_rn(-static_cast<float>(mc.s), f1[e], uh);
     }

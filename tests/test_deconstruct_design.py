@@ -166,13 +166,17 @@ def test_limb_sum_stays_in_range_at_the_extremes(m):
 
 
 def square_digits_fp(u, s, h0, h1):
-    """The kernel's FP32 digits of u = c + h0 + s·h1 for s ≠ 32: the float
-    1.5·2^23 + u, one fused multiply-add rounded down,
-    t = 1.5·2^23 + ⌊u·⌈2^17/s⌉/2^17⌋ (exact: the grid at 1.5·2^23 is the
-    integers), d1 = t - (1.5·2^23 + h1), d0 = (u - h0 - s·h1) - s·d1."""
+    """The kernel's FP32 digits of u = c + h0 + s·h1 for s ≠ 32: with the
+    float ub = 1.5·2^23 + u and cs = ⌈2^17/s⌉/2^17, one fused multiply-add
+    rounded down, t = RD(ub·cs + (1.5·2^23 - 96·⌈2^17/s⌉)), which is
+    1.5·2^23 + ⌊u·⌈2^17/s⌉/2^17⌋ (the grid at 1.5·2^23 is the integers);
+    d1 = t - (1.5·2^23 + h1), d0 = (u - h0 - s·h1) - s·d1."""
     c17 = -(-(1 << 17) // s)
     base = 3 << 22
-    t = base + (u * c17) // (1 << 17)
+    addend = base - 96 * c17
+    assert 0 < addend < 1 << 24 and 96 * c17 * (1 << 17) == base * c17   # 1.5·2^23·cs = 96·c17
+    ub = base + np.asarray(u, dtype=object)
+    t = np.array([(int(x) * c17 + addend * (1 << 17)) // (1 << 17) for x in ub], dtype=np.int64)  # RD of the exact value
     d1 = t - (base + h1)
     d0 = (u - h0 - s * h1) - s * d1
     return d0, d1, t
