@@ -19,7 +19,6 @@ constexpr int kFT = 64, kFK = 16;
 __global__ void compact_flags_kernel(int64_t m, int64_t n, const uint8_t* __restrict__ row_flag,
                                      const uint8_t* __restrict__ col_flag, int* __restrict__ row_list,
                                      int* __restrict__ col_list, int* __restrict__ count) {
-  pdl_trigger();  // the FMA kernel may be scheduled now; it waits for the lists
   const bool cols = blockIdx.y == 1;
   const int64_t cnt = cols ? n : m;
   const uint8_t* flag = cols ? col_flag : row_flag;
@@ -42,7 +41,6 @@ __global__ void __launch_bounds__(256) fma_gemm_kernel(int64_t m, int64_t n, int
   __shared__ double As[kFK][kFT + 1];
   __shared__ double Bs[kFK][kFT + 1];
   __shared__ int rid[kFT], cid[kFT];
-  pdl_wait();  // the lists and counts are complete (a no-op when launched plainly)
   if (gridDim.y == 2) {
     if (blockIdx.y == 0) {
       col_list = nullptr;
@@ -135,12 +133,10 @@ cudaError_t launch_fallback_lists(int64_t m, int64_t n, int64_t k, const double*
   const int64_t most = m > n ? m : n;
   const unsigned cg = static_cast<unsigned>(std::min<int64_t>((most + 255) / 256, 4096));
   compact_flags_kernel<<<dim3(cg, 2), 256, 0, st>>>(m, n, row_flag, col_flag, rlist, clist, counts);
-  // flagged rows × all columns (blockIdx.y = 0), all rows × flagged columns
-  // (1), scheduled while the compaction finishes
-  const cudaError_t err = launch_dependent(fma_gemm_kernel, dim3(fb_grid(), 2), dim3(256), 0, st, m, n, k, A, lda, B,
-                                           ldb, static_cast<const int*>(rlist), static_cast<const int*>(counts),
-                                           static_cast<const int*>(clist), static_cast<const int*>(counts + 1), C, ldc);
-  return err != cudaSuccess ? err : cudaGetLastError();
+  // flagged rows × all columns (blockIdx.y = 0), all rows × flagged columns (1)
+  fma_gemm_kernel<<<dim3(fb_grid(), 2), 256, 0, st>>>(m, n, k, A, lda, B, ldb, rlist, counts, clist, counts + 1, C,
+                                                       ldc);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_native(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, const double* B,
