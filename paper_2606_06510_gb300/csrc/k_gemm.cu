@@ -351,10 +351,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           if (c == 48 && !carry) {
             // The last chunk is in registers: release the accumulators now,
             // so the next unit's MMAs overlap this chunk's reduction and
-            // stores.
+            // stores.  The arrive is relaxed: the residue stores before it
+            // need no ordering against the MMAs, and a release would wait
+            // for them to be performed.
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive_remote(acc_empty_leader);
+            if (lane == 0) mbar_arrive_remote_relaxed(acc_empty_leader);
           }
           if (MODE == 1) {
 #pragma unroll

@@ -266,6 +266,15 @@ __device__ __forceinline__ void cluster_sync_all() {
 __device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr) {
   asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
 }
+// The same arrive without release semantics: it orders none of the thread's
+// earlier memory operations (a release would hold the arrive until the
+// thread's outstanding global stores are performed).  For a thread whose
+// tensor-memory loads have completed (tcgen05.wait::ld, then
+// tcgen05.fence::before_thread_sync), program order alone puts those loads
+// before the arrive.
+__device__ __forceinline__ void mbar_arrive_remote_relaxed(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
 // 3-D tiled TMA load issued by either CTA of a pair; the transaction bytes
 // complete on `bar` (a shared::cluster address, here the leader CTA's barrier).
 __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap* map, uint32_t bar, int x, int y) {
