@@ -124,13 +124,15 @@ int oz2_dgemm(int64_t m, int64_t n, int64_t k,
  * back, and synchronises `stream` before returning.  Device buffers and the
  * workspace are allocated and freed stream-ordered inside the call, from the
  * library's memory pool.  A contiguous matrix (ld = rows) moves in one
- * linear copy, any other in a pitched copy.  For wide C (n ≥ 1536) the
- * residue GEMM, reconstruction and fallback run by column blocks (a last
- * block of 256 columns; at most 8 blocks, the others multiples of 256 wide
- * chosen to fill the GEMM's last wave), and each block of C
- * is copied back on a library-owned copy stream while the next block is
- * computed; the result is the same as unblocked.  Host-buffer calls on one
- * device share that stream and are serialised. */
+ * linear copy, any other in a pitched copy.  The copies run on a
+ * library-owned copy stream: B first, then A in up to 4 column chunks (of
+ * at least 32 MB); B's scan, flags and magnitude planes run while A is
+ * copied, and A's scan chunk by chunk as its columns arrive.  The residue
+ * GEMM, reconstruction and fallback then run by column blocks (oz2_plan's
+ * host_widths), and each block of C is copied back on the copy stream while
+ * the next block is computed.  The result is the same as one oz2_dgemm on
+ * device copies.  Host-buffer calls on one device share the copy stream and
+ * are serialised. */
 int oz2_dgemm_host(int64_t m, int64_t n, int64_t k,
                    const double* h_A, int64_t lda,
                    const double* h_B, int64_t ldb,
@@ -223,8 +225,14 @@ int oz2_workspace_layout(int64_t m, int64_t n, int64_t k, int num_moduli,
  *   host_blocks   column blocks of oz2_dgemm_host (1 to 8).  The blocks run
  *                 the residue GEMM, reconstruction and fallback one after
  *                 another, each copied back while the next computes.
- *   host_widths   their widths: multiples of 256 but the last, which is
- *                 the last (possibly ragged) 256-column tile column.
+ *   host_widths   their widths: multiples of 256 but the last.  They
+ *                 minimise the end of the last copy back on a model of the
+ *                 call: each block's GEMM waves and reconstruction at this
+ *                 library's rates on a GB300, its copy at 190 GB/s over the
+ *                 host link, one copy at a time.  Long k gives a narrow last
+ *                 block (its copy is the one left exposed); short k, where
+ *                 the copies dominate, a narrow first one (the copies start
+ *                 early).  Identical shapes reuse the last plan.
  *   host_kparts   the residue GEMM's kparts for each block.
  * Returns OZ2_OK, OZ2_ERR_INVALID_ARG (null out, negative sizes,
  * cta_pairs < 1) or OZ2_ERR_UNSUPPORTED_R. */

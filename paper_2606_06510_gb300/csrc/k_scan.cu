@@ -3,7 +3,7 @@
 // fallback flags, and the choice of D and E from the "+1" pass (§2.4).
 #include <climits>
 
-#include "oz2_common.cuh"
+#include "k_scan.cuh"
 
 namespace oz2 {
 
@@ -100,8 +100,8 @@ __global__ void __launch_bounds__(256) scan_kernel(int64_t m, int64_t n, int64_t
   }
 }
 
-// One block per operand (0: rows of A, 1: columns of B).  Decodes the scan
-// keys, finds the lower median of the exponents of the nonzero finite rows,
+// One block per operand (block b takes operand first_op + b; 0: rows of A,
+// 1: columns of B).  Decodes the scan keys, finds the lower median of the exponents of the nonzero finite rows,
 // and writes the flags (bit0: native fallback; bit1: zero in the emulation)
 // and the final exponent (0 for rows that are zero in the emulation).
 constexpr int kExpBins = 2112;   // frexp exponents of finite doubles: [-1073, 1024]
@@ -112,13 +112,13 @@ constexpr int kBinsPerThread = (kExpBins + kFinalizeThreads - 1) / kFinalizeThre
 __global__ void __launch_bounds__(kFinalizeThreads) finalize_flags_kernel(int64_t m, int64_t n, int* __restrict__ ra,
                                       int* __restrict__ cb, uint8_t* __restrict__ row_flag,
                                       uint8_t* __restrict__ col_flag, unsigned flags,
-                                      Oz2Device* dev) {
+                                      Oz2Device* dev, int first_op) {
   __shared__ int hist[kExpBins];
   __shared__ int warp_sum[32];
   __shared__ int med_s;
   __shared__ int count_s;
   pdl_wait();  // the scan keys are complete
-  const bool is_a = blockIdx.x == 0;
+  const bool is_a = blockIdx.x + first_op == 0;
   const int64_t cnt = is_a ? m : n;
   int* key = is_a ? ra : cb;
   uint8_t* fl = is_a ? row_flag : col_flag;
@@ -198,6 +198,44 @@ __global__ void __launch_bounds__(kFinalizeThreads) finalize_flags_kernel(int64_
   }
 }
 
+cudaError_t launch_scan_keys(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, const double* B,
+                             int64_t ldb, ScanOut out, cudaStream_t st) {
+  if (k <= 0 || (m <= 0 && n <= 0)) return cudaSuccess;
+  ScanGrid g{};
+  g.achunk = 64;
+  int64_t ks = (k + g.achunk - 1) / g.achunk;
+  if (ks > 65535) {
+    g.achunk = static_cast<int>((k + 65534) / 65535);
+    ks = (k + g.achunk - 1) / g.achunk;
+  }
+  g.bchunk = 1024;
+  int64_t bks = (k + g.bchunk - 1) / g.bchunk;
+  if (bks > 65535) {
+    g.bchunk = static_cast<int>((k + 65534) / 65535 + 1) & ~1;
+    bks = (k + g.bchunk - 1) / g.bchunk;
+  }
+  g.gax = (m + 255) / 256;
+  g.ga = m > 0 ? g.gax * ks : 0;
+  g.gbx = (n + 7) / 8;
+  const int64_t gb = n > 0 ? g.gbx * bks : 0;
+  g.vec = (ldb % 2 == 0) && (reinterpret_cast<uintptr_t>(B) % 16 == 0);
+  if (g.ga + gb > 0x7FFFFFFFLL) return cudaErrorInvalidValue;
+  count_launch();
+  scan_kernel<<<static_cast<unsigned>(g.ga + gb), 256, 0, st>>>(m, n, k, A, lda, B, ldb, g, out.ra, out.cb);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_scan_flags(int64_t m, int64_t n, int ops, unsigned flags, ScanOut out, Oz2Device* dev,
+                              cudaStream_t st) {
+  if ((ops & 3) == 0) return cudaSuccess;
+  const int first = (ops & 1) ? 0 : 1;
+  const int count = ops == 3 ? 2 : 1;
+  count_launch();
+  const cudaError_t e = launch_dependent(finalize_flags_kernel, dim3(count), dim3(kFinalizeThreads), 0, st, m, n,
+                                         out.ra, out.cb, out.row_flag, out.col_flag, flags, dev, first);
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
+
 cudaError_t launch_scan(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda,
                         const double* B, int64_t ldb, unsigned flags, ScanOut out,
                         Oz2Device* dev, cudaStream_t st, bool zero_keys) {
@@ -205,33 +243,8 @@ cudaError_t launch_scan(int64_t m, int64_t n, int64_t k, const double* A, int64_
   // The scan keys are maxima taken with atomics: zero unless the caller has.
   if (zero_keys && m > 0 && (err = cudaMemsetAsync(out.ra, 0, sizeof(int) * m, st)) != cudaSuccess) return err;
   if (zero_keys && n > 0 && (err = cudaMemsetAsync(out.cb, 0, sizeof(int) * n, st)) != cudaSuccess) return err;
-  if (k > 0 && (m > 0 || n > 0)) {
-    ScanGrid g{};
-    g.achunk = 64;
-    int64_t ks = (k + g.achunk - 1) / g.achunk;
-    if (ks > 65535) {
-      g.achunk = static_cast<int>((k + 65534) / 65535);
-      ks = (k + g.achunk - 1) / g.achunk;
-    }
-    g.bchunk = 1024;
-    int64_t bks = (k + g.bchunk - 1) / g.bchunk;
-    if (bks > 65535) {
-      g.bchunk = static_cast<int>((k + 65534) / 65535 + 1) & ~1;
-      bks = (k + g.bchunk - 1) / g.bchunk;
-    }
-    g.gax = (m + 255) / 256;
-    g.ga = m > 0 ? g.gax * ks : 0;
-    g.gbx = (n + 7) / 8;
-    const int64_t gb = n > 0 ? g.gbx * bks : 0;
-    g.vec = (ldb % 2 == 0) && (reinterpret_cast<uintptr_t>(B) % 16 == 0);
-    if (g.ga + gb > 0x7FFFFFFFLL) return cudaErrorInvalidValue;
-    count_launch();
-    scan_kernel<<<static_cast<unsigned>(g.ga + gb), 256, 0, st>>>(m, n, k, A, lda, B, ldb, g, out.ra, out.cb);
-  }
-  count_launch();
-  const cudaError_t e2 = launch_dependent(finalize_flags_kernel, dim3(2), dim3(kFinalizeThreads), 0, st, m, n, out.ra,
-                                          out.cb, out.row_flag, out.col_flag, flags, dev);
-  return e2 != cudaSuccess ? e2 : cudaGetLastError();
+  if ((err = launch_scan_keys(m, n, k, A, lda, B, ldb, out, st)) != cudaSuccess) return err;
+  return launch_scan_flags(m, n, 3, flags, out, dev, st);
 }
 
 // ---------------------------------------------------------------------------

@@ -9,8 +9,9 @@
 #include <cstring>
 #include <functional>
 #include <mutex>
+#include <vector>
 
-#include "oz2_common.cuh"
+#include "k_scan.cuh"
 
 namespace oz2 {
 
@@ -20,6 +21,7 @@ static const int kModuliAll[kMaxModuli] = {1089, 1024, 961, 841, 625, 529, 511, 
                                            503,  499,  491, 487, 479, 467, 463, 461};
 constexpr int kTableMax = 20480;  // 2·Σ of the ten nonsquare moduli = 9740 entries
 constexpr int kHostBlocksMax = 8;   // column blocks of one oz2_dgemm_host call
+constexpr int kHostAChunksMax = 4;  // column chunks A is copied in by oz2_dgemm_host
 
 // Packed E4M3 digit planes of every residue (byte p = plane p) of the
 // nonsquare moduli, 2m entries per modulus, entry i for the residue
@@ -244,11 +246,15 @@ struct DeviceState {
   // allocates, so entry points that allocate nothing never create it.
   cudaMemPool_t pool = nullptr;
   bool pool_tried = false;
-  // oz2_dgemm_host: a stream for copying finished column blocks of C back,
-  // one event per block and one for the last copy, created on first use; the
-  // mutex serialises host-buffer calls on this device, which share them.
+  // oz2_dgemm_host: a stream for the copies (A and B in, then the finished
+  // column blocks of C back), one event for the staging buffer's
+  // allocation, one per arrived part of the operands, one per block and one
+  // for the last copy, created on first use; the mutex serialises
+  // host-buffer calls on this device, which share them.
   std::mutex host_mu;
   cudaStream_t copy_stream = nullptr;
+  cudaEvent_t staged = nullptr;
+  cudaEvent_t arrived[1 + kHostAChunksMax] = {};
   cudaEvent_t block_done[kHostBlocksMax] = {};
   cudaEvent_t copies_done = nullptr;
 };
@@ -501,14 +507,27 @@ struct ColumnBlocks {
   int64_t widths[kHostBlocksMax] = {};
 };
 
+// Operands that arrive on another stream while phase 1 runs (oz2_dgemm_host):
+// B whole when b_ready has completed, then A by column chunks, columns
+// [a_col0[c], a_col0[c + 1]) when a_ready[c] has.
+struct Arrivals {
+  cudaEvent_t b_ready = nullptr;
+  int a_chunks = 0;
+  int64_t a_col0[kHostAChunksMax + 1] = {};
+  cudaEvent_t a_ready[kHostAChunksMax] = {};
+};
+
 // Algorithm 1 on the call's stream.  Phase 1 (scan, "+1" pass, scales,
 // deconstruction) covers the whole problem; the residue GEMM, the
 // reconstruction and the fallback then run per column block (all of C when
-// `blocks` is null), each followed by `on_block`.  The results do not depend
-// on the blocking.
+// `blocks` is null), each followed by `on_block`.  With `in`, the operands
+// are still arriving: B's scan, flags and magnitude planes run as soon as B
+// is in, and A's scan chunk by chunk as its columns come (the row keys are
+// maxima, merged across chunks).  The results depend on neither.
 static int run_stages(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, const double* B, int64_t ldb,
                       double* C, int64_t ldc, int num_moduli, int quant, int scale, unsigned flags, void* workspace,
-                      size_t ws_bytes, void* stream, const ColumnBlocks* blocks, const BlockDone* on_block) {
+                      size_t ws_bytes, void* stream, const ColumnBlocks* blocks, const BlockDone* on_block,
+                      const Arrivals* in = nullptr) {
   int st = check_sizes(m, n, k, lda, ldb, ldc);
   if (st) return st;
   if (num_moduli < 1 || num_moduli > kMaxModuli) return OZ2_ERR_UNSUPPORTED_R;
@@ -576,12 +595,27 @@ static int run_stages(int64_t m, int64_t n, int64_t k, const double* A, int64_t 
                                                                                               n, urow, misc);
   }
   mark(0);
-  if (err == cudaSuccess)
-    err = launch_scan(m, n, k, A, lda, B, ldb, flags, ScanOut{ra, cb, rf, cf}, ds->status, s, false);
+  const ScanOut so{ra, cb, rf, cf};
+  if (in) {
+    if (err == cudaSuccess) err = cudaStreamWaitEvent(s, in->b_ready, 0);
+    if (err == cudaSuccess) err = launch_scan_keys(0, n, k, nullptr, lda, B, ldb, so, s);
+    if (err == cudaSuccess) err = launch_scan_flags(m, n, 2, flags, so, ds->status, s);
+    if (err == cudaSuccess && scale == OZ2_SCALE_R2)
+      err = launch_magnitude_planes(0, n, k, A, lda, B, ldb, ra, cb, rf, cf, mag_a, mag_b, s);
+    for (int c = 0; c < in->a_chunks && err == cudaSuccess; ++c) {
+      err = cudaStreamWaitEvent(s, in->a_ready[c], 0);
+      const int64_t k0 = in->a_col0[c];
+      if (err == cudaSuccess)
+        err = launch_scan_keys(m, 0, in->a_col0[c + 1] - k0, A + k0 * lda, lda, nullptr, ldb, so, s);
+    }
+    if (err == cudaSuccess) err = launch_scan_flags(m, n, 1, flags, so, ds->status, s);
+  } else if (err == cudaSuccess) {
+    err = launch_scan(m, n, k, A, lda, B, ldb, flags, so, ds->status, s, false);
+  }
   mark(1);
   if (scale == OZ2_SCALE_R2) {
     if (err == cudaSuccess)
-      err = launch_magnitude_planes(m, n, k, A, lda, B, ldb, ra, cb, rf, cf, mag_a, mag_b, s);
+      err = launch_magnitude_planes(m, in ? 0 : n, k, A, lda, B, ldb, ra, cb, rf, cf, mag_a, mag_b, s);
     mark(2);
     if (err == cudaSuccess)
       err = launch_plane_gemm(m, n, L.k_pad, mods, mag_a, mag_b, simt ? 3 : 1, nullptr, 0, urow, ds->status, s);
@@ -643,46 +677,136 @@ int oz2_dgemm_ex(int64_t m, int64_t n, int64_t k, const double* A, int64_t lda, 
                     nullptr, nullptr);
 }
 
-// Column blocks for oz2_dgemm_host.  C's copy back overlaps the blocks after
-// the one copied, so the last block's copy is exposed: it is one 256-column
-// tile column.  The others take c tile columns each, c from the smallest
-// width that stays within the block budget up to three more, chosen so that
-// the residue GEMM's units (⌈m/256⌉·r per tile column) fill the last wave
-// over its persistent CTA pairs as fully as possible.  Narrow C (n < 1536)
-// is one block.
-static ColumnBlocks host_column_blocks(int64_t m, int64_t n, int r, int64_t pairs) {
+// Column blocks for oz2_dgemm_host, chosen on a model of the call's second
+// phase.  Block i's residue GEMM takes ⌈u_i/P⌉ waves of one unit's time
+// (u_i = ⌈m/256⌉·r units per tile column of the block, P CTA pairs), its
+// reconstruction moves m·(2r + 8) bytes of HBM per column, and its copy back
+// moves 8m bytes per column over the host link, on one stream, once the
+// block is done and the copy before it has finished.  Among the partitions
+// into at most kHostBlocksMax blocks of whole tile columns (or of groups of
+// them, when C has more than 64), the one whose last copy ends first is
+// taken, by dynamic programming over the Pareto front of (end of compute,
+// end of copies) after each prefix of the columns.  A small first block
+// starts the copies early when the link is the bottleneck (short k); a
+// small last block leaves little copy exposed when the GPU is (long k).
+// The rates are this kernel's, measured on one GB300 and its host link.
+namespace {
+constexpr double kModelPairFlops = 46e12;     // residue GEMM, FP8 flop/s per CTA pair
+constexpr double kModelUnitExtra = 2e-6;      // per unit: the accumulator drain
+constexpr double kModelCrtBytes = 4.0e12;     // reconstruction, bytes/s
+constexpr double kModelLink = 190e9;          // device to pinned host, bytes/s
+constexpr double kModelBlockExtra = 8e-6;     // per block: its launches
+constexpr double kModelCopyExtra = 5e-6;      // per copy
+constexpr int kModelGroupsMax = 64;
+
+struct BlockModel {
+  int64_t m, n, tiles, per_tile, pairs, group;
+  double t_unit, crt_per_col, d2h_per_col;
+  int64_t cols(int64_t g0, int64_t g1) const {
+    return std::min(n, g1 * group * 256) - std::min(n, g0 * group * 256);
+  }
+  double compute(int64_t g0, int64_t g1) const {
+    const int64_t t = std::min(tiles, g1 * group) - g0 * group;
+    const int64_t waves = (per_tile * t + pairs - 1) / pairs;
+    return static_cast<double>(waves) * t_unit + static_cast<double>(cols(g0, g1)) * crt_per_col +
+           kModelBlockExtra;
+  }
+  double copy(int64_t g0, int64_t g1) const { return static_cast<double>(cols(g0, g1)) * d2h_per_col + kModelCopyExtra; }
+};
+
+struct ModelState {
+  double ce, cp;    // end of the blocks' compute, end of their copies
+  int64_t g;        // groups covered
+  int parent;       // index in the previous layer's front for g's predecessor
+  int64_t from;     // first group of the last block
+};
+}  // namespace
+
+static ColumnBlocks plan_column_blocks(int64_t m, int64_t n, int r, int64_t k, int64_t pairs) {
   ColumnBlocks b;
   const int64_t tiles = (n + 255) / 256;
-  if (n < 1536 || tiles < 4) {
+  if (tiles < 2 || m == 0 || k == 0) {
     b.count = 1;
     b.widths[0] = n;
     return b;
   }
-  const int64_t per_tile = (m + 255) / 256 * r;
-  int64_t left = tiles - 1;  // tile columns before the last
-  while (left > 0) {
-    const int64_t slots = kHostBlocksMax - 1 - b.count;  // blocks left before the last one
-    int64_t best_c = left;
-    if (slots > 1) {
-      const int64_t c_min = std::max<int64_t>(3, (left + slots - 1) / slots);
-      double best_idle = 2.0;
-      best_c = std::min(left, c_min);
-      for (int64_t c = c_min; c < c_min + 4 && c <= left; ++c) {
-        const int64_t rest = left - c;
-        if (rest != 0 && rest < 3 && rest < c_min) continue;  // no sliver before the last block
-        const double waves = static_cast<double>(per_tile * c) / static_cast<double>(pairs);
-        const double idle = (std::ceil(waves) - waves) / std::ceil(waves);  // idle share of the launch
-        if (idle < best_idle - 1e-9) {
-          best_idle = idle;
-          best_c = c;
-        }
+  BlockModel M;
+  M.m = m;
+  M.n = n;
+  M.tiles = tiles;
+  M.per_tile = (m + 255) / 256 * r;
+  M.pairs = std::max<int64_t>(1, pairs);
+  M.group = (tiles + kModelGroupsMax - 1) / kModelGroupsMax;
+  const int64_t k_pad = (k + kKPad - 1) / kKPad * kKPad;
+  M.t_unit = 3.0 * 2.0 * 256.0 * 256.0 * static_cast<double>(k_pad) / kModelPairFlops + kModelUnitExtra;
+  M.crt_per_col = static_cast<double>(m) * (2.0 * r + 8.0) / kModelCrtBytes;
+  M.d2h_per_col = static_cast<double>(m) * 8.0 / kModelLink;
+  const int64_t G = (tiles + M.group - 1) / M.group;
+  // fronts[j][g]: partitions of the first g groups into j blocks.
+  std::vector<std::vector<std::vector<ModelState>>> fronts(
+      kHostBlocksMax + 1, std::vector<std::vector<ModelState>>(G + 1));
+  fronts[0][0].push_back(ModelState{0.0, 0.0, 0, -1, 0});
+  double best = 1e300;
+  int best_j = 0, best_i = 0;
+  for (int j = 0; j <= kHostBlocksMax; ++j) {
+    for (int64_t g = 0; g <= G; ++g) {
+      std::vector<ModelState>& f = fronts[j][g];
+      if (f.empty()) continue;
+      // Keep the Pareto front: by compute end, then strictly falling copy end.
+      std::sort(f.begin(), f.end(), [](const ModelState& x, const ModelState& y) {
+        return x.ce < y.ce || (x.ce == y.ce && x.cp < y.cp);
+      });
+      std::vector<ModelState> kept;
+      for (const ModelState& x : f)
+        if (kept.empty() || x.cp < kept.back().cp) kept.push_back(x);
+      f.swap(kept);
+      if (g == G) {
+        for (int i = 0; i < static_cast<int>(f.size()); ++i)
+          if (f[i].cp < best - 1e-12) {
+            best = f[i].cp;
+            best_j = j;
+            best_i = i;
+          }
+        continue;
       }
+      if (j == kHostBlocksMax) continue;
+      for (int i = 0; i < static_cast<int>(f.size()); ++i)
+        for (int64_t g1 = g + 1; g1 <= G; ++g1) {
+          const double ce = f[i].ce + M.compute(g, g1);
+          const double cp = std::max(ce, f[i].cp) + M.copy(g, g1);
+          fronts[j + 1][g1].push_back(ModelState{ce, cp, g1, i, g});
+        }
     }
-    b.widths[b.count++] = best_c * 256;
-    left -= best_c;
   }
-  b.widths[b.count++] = n - 256 * (tiles - 1);  // the last (possibly ragged) tile column
+  // Walk back from the best complete partition.
+  int64_t widths[kHostBlocksMax];
+  int j = best_j, i = best_i;
+  int64_t g = G;
+  while (j > 0) {
+    const ModelState& x = fronts[j][g][i];
+    widths[j - 1] = M.cols(x.from, g);
+    i = x.parent;
+    g = x.from;
+    --j;
+  }
+  b.count = best_j;
+  for (int q = 0; q < best_j; ++q) b.widths[q] = widths[q];
   return b;
+}
+
+// The plan of the last shape asked for is kept: a loop of calls on one shape
+// plans once (a plan over many tile columns takes a few milliseconds).
+static ColumnBlocks host_column_blocks(int64_t m, int64_t n, int r, int64_t k, int64_t pairs) {
+  static std::mutex mu;
+  static int64_t key[5] = {-1, -1, -1, -1, -1};
+  static ColumnBlocks cached;
+  const int64_t want[5] = {m, n, static_cast<int64_t>(r), k, pairs};
+  std::lock_guard<std::mutex> lk(mu);
+  if (!std::equal(want, want + 5, key)) {
+    cached = plan_column_blocks(m, n, r, k, pairs);
+    std::copy(want, want + 5, key);
+  }
+  return cached;
 }
 
 int oz2_plan(int64_t m, int64_t n, int64_t k, int num_moduli, int cta_pairs, oz2_plan_info* out) {
@@ -698,7 +822,7 @@ int oz2_plan(int64_t m, int64_t n, int64_t k, int num_moduli, int cta_pairs, oz2
                                L.planes_a - L.mag_a, cta_pairs);
   };
   out->kparts = kparts(n);
-  const ColumnBlocks b = host_column_blocks(m, n, num_moduli, cta_pairs);
+  const ColumnBlocks b = host_column_blocks(m, n, num_moduli, k, cta_pairs);
   out->host_blocks = b.count;
   for (int i = 0; i < b.count; ++i) {
     out->host_widths[i] = b.widths[i];
@@ -740,9 +864,13 @@ int oz2_dgemm_host(int64_t m, int64_t n, int64_t k, const double* hA, int64_t ld
   std::lock_guard<std::mutex> host_lock(ds->host_mu);
   if (!ds->copy_stream) {
     if (cudaStreamCreateWithFlags(&ds->copy_stream, cudaStreamNonBlocking) != cudaSuccess) return OZ2_ERR_CUDA;
-    for (int i = 0; i < kHostBlocksMax; ++i)
-      if (cudaEventCreateWithFlags(&ds->block_done[i], cudaEventDisableTiming) != cudaSuccess) return OZ2_ERR_CUDA;
-    if (cudaEventCreateWithFlags(&ds->copies_done, cudaEventDisableTiming) != cudaSuccess) return OZ2_ERR_CUDA;
+    bool ok = cudaEventCreateWithFlags(&ds->staged, cudaEventDisableTiming) == cudaSuccess &&
+              cudaEventCreateWithFlags(&ds->copies_done, cudaEventDisableTiming) == cudaSuccess;
+    for (int i = 0; ok && i < 1 + kHostAChunksMax; ++i)
+      ok = cudaEventCreateWithFlags(&ds->arrived[i], cudaEventDisableTiming) == cudaSuccess;
+    for (int i = 0; ok && i < kHostBlocksMax; ++i)
+      ok = cudaEventCreateWithFlags(&ds->block_done[i], cudaEventDisableTiming) == cudaSuccess;
+    if (!ok) return OZ2_ERR_CUDA;
   }
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaStream_t cs = ds->copy_stream;
@@ -757,10 +885,27 @@ int oz2_dgemm_host(int64_t m, int64_t n, int64_t k, const double* hA, int64_t ld
   double* dA = reinterpret_cast<double*>(buf);
   double* dB = reinterpret_cast<double*>(buf + bA);
   double* dC = reinterpret_cast<double*>(buf + bA + bB);
-  cudaError_t err = cudaSuccess;
-  if (k > 0) {
-    err = copy_matrix(dA, m, hA, lda, m, k, cudaMemcpyHostToDevice, s);
-    if (err == cudaSuccess) err = copy_matrix(dB, k, hB, ldb, k, n, cudaMemcpyHostToDevice, s);
+  // Every copy runs on the copy stream, after the staging buffer exists: B
+  // first, then A by column chunks (of at least 32 MB, multiples of 64
+  // columns), each marked by an event that the call's stream waits on
+  // before the scan of that part (phase 1 overlaps the copies).
+  cudaError_t err = cudaEventRecord(ds->staged, s);
+  if (err == cudaSuccess) err = cudaStreamWaitEvent(cs, ds->staged, 0);
+  Arrivals in;
+  if (k > 0 && err == cudaSuccess) {
+    err = copy_matrix(dB, k, hB, ldb, k, n, cudaMemcpyHostToDevice, cs);
+    if (err == cudaSuccess) err = cudaEventRecord(ds->arrived[0], cs);
+    in.b_ready = ds->arrived[0];
+    const int64_t want = std::min<int64_t>(kHostAChunksMax, std::max<int64_t>(1, static_cast<int64_t>(bA >> 25)));
+    const int64_t step = std::max<int64_t>(64, (k + want - 1) / want + 63) / 64 * 64;
+    for (int64_t k0 = 0; k0 < k && err == cudaSuccess; k0 += step) {
+      const int64_t kc = std::min(step, k - k0);
+      err = copy_matrix(dA + k0 * m, m, hA + k0 * lda, lda, m, kc, cudaMemcpyHostToDevice, cs);
+      if (err == cudaSuccess) err = cudaEventRecord(ds->arrived[1 + in.a_chunks], cs);
+      in.a_ready[in.a_chunks] = ds->arrived[1 + in.a_chunks];
+      in.a_col0[in.a_chunks++] = k0;
+      in.a_col0[in.a_chunks] = k0 + kc;
+    }
   }
   // C goes back by column blocks on the copy stream, each as soon as its
   // reconstruction and fallback are done, so that the copies overlap the
@@ -768,7 +913,7 @@ int oz2_dgemm_host(int64_t m, int64_t n, int64_t k, const double* hA, int64_t ld
   int dev = 0, sms = 148;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  const ColumnBlocks blocks = host_column_blocks(m, n, num_moduli, std::max(1, sms / 2));
+  const ColumnBlocks blocks = host_column_blocks(m, n, num_moduli, k, std::max(1, sms / 2));
   int blk = 0;
   const BlockDone copy_back = [&](int64_t c0, int64_t cols) -> cudaError_t {
     cudaError_t e = cudaEventRecord(ds->block_done[blk], s);
@@ -780,7 +925,7 @@ int oz2_dgemm_host(int64_t m, int64_t n, int64_t k, const double* hA, int64_t ld
   if (err == cudaSuccess) {
     if (k > 0) {
       st = run_stages(m, n, k, dA, m, dB, k, dC, m, num_moduli, OZ2_QUANT_TZ, OZ2_SCALE_R2, 0,
-                      buf + bA + bB + bC, ws, stream, &blocks, &copy_back);
+                      buf + bA + bB + bC, ws, stream, &blocks, &copy_back, &in);
     } else {  // C = 0
       err = cudaMemsetAsync(dC, 0, sizeof(double) * m * n, s);
       if (err == cudaSuccess) err = copy_back(0, n);

@@ -114,6 +114,7 @@ def check_full_size(oz, A, B, r, rows, cols):
                 assert bound <= 2 ** T
                 want = orc.unscale_one(exact_dot(At[a], Bt[b]), -int(d[i] + e[j]))
             assert got == want and np.signbit(got) == np.signbit(want), (i, j, got, want)
+    return C
 
 
 def sample_cols(n, count, seed):

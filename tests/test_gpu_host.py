@@ -1,8 +1,11 @@
 """The host-buffer entry oz2_dgemm_host against the CPU oracle, bit for bit.
 
-For wide C the entry runs the residue GEMM, the reconstruction and the
-fallback by column blocks of about 1024 columns and copies each block of C
-back while the next one is computed; the result must not depend on that.
+The entry copies B in, then A by column chunks (four of at least 32 MB for
+A of 128 MB or more), while the scan of each arrived part runs; the row keys
+of A are maxima merged across its chunks.  It then runs the residue GEMM,
+the reconstruction and the fallback by column blocks (oz2_plan's
+host_widths) and copies each block of C back while the next one is
+computed.  The result must depend on neither.
 """
 import numpy as np
 import pytest
@@ -10,6 +13,7 @@ import pytest
 import workloads as wl
 from helpers import ensure_built
 from oracle import ozaki2 as orc
+from test_gpu_full_size import check_full_size, sample_cols
 
 pytestmark = pytest.mark.gpu
 
@@ -40,16 +44,18 @@ def assert_same(got, want):
 
 
 def test_column_blocks_with_fallback_and_padded_c(oz):
-    """n = 2600: blocks of 1024, 1024 and 552 columns.  A fallback row (2^300)
-    and a zero row in A; a NaN column in the second block and a 2^-200 column
-    in the last one; C with leading dimension m + 5."""
+    """n = 2600: blocks of 1280 and 1320 columns.  A fallback row (2^300)
+    and a zero row in A; a NaN column in each block's range and a 2^-200
+    column at the end; C with leading dimension m + 5."""
     import torch
     m, n, k = 300, 2600, 70
+    assert oz.oz2_plan(m, n, k, 12)["host_widths"] == [1280, 1320]
     A = np.array(wl.random_matrix(m, k, 1.0, 7100), order="F")
     B = np.array(wl.random_matrix(k, n, 1.0, 7200), order="F")
     A[7, :] *= 2.0 ** 300
     A[123, :] = 0.0
     B[3, 1500] = np.nan
+    B[5, 40] = np.nan
     B[:, 2599] *= 2.0 ** -200
     want = orc.oz2_dgemm(A, B, 12).C
     C = torch.full((n, m + 5), 7.0, dtype=torch.float64, pin_memory=True).t()[:m]
@@ -77,14 +83,19 @@ def test_empty_k_gives_zero(oz):
 
 @pytest.mark.parametrize("seed", range(4))
 def test_randomised_wide_problems(oz, seed):
-    """Seeded wide problems (n from 1400 to 3400, so two to three column
-    blocks with a ragged last one), r from 1 to 16, φ from 0 to 5, and
-    planted special rows of A and columns of B in random blocks."""
+    """Seeded wide problems (n from 1400 to 3400, drawn until the plan has
+    at least two column blocks, the last one ragged), r from 1 to 16, φ from
+    0 to 5, and planted special rows of A and columns of B in random
+    blocks."""
     rng = np.random.default_rng(8000 + seed)
-    m = int(rng.integers(1, 200))
-    n = int(rng.integers(1400, 3400))
-    k = int(rng.integers(1, 120))
-    r = int(rng.integers(1, 17))
+    for _ in range(100):
+        m = int(rng.integers(150, 500))
+        n = int(rng.integers(1400, 3400))
+        k = int(rng.integers(1, 120))
+        r = int(rng.integers(1, 17))
+        if len(oz.oz2_plan(m, n, k, r)["host_widths"]) >= 2:
+            break
+    assert len(oz.oz2_plan(m, n, k, r)["host_widths"]) >= 2
     phi = float(rng.uniform(0.0, 5.0))
     A = np.array(wl.random_matrix(m, k, phi, 8100 + seed), order="F")
     B = np.array(wl.random_matrix(k, n, phi, 8200 + seed), order="F")
@@ -107,15 +118,40 @@ def test_randomised_wide_problems(oz, seed):
 
 def test_column_blocks_with_split_k(oz):
     """A short C with a long k: each column block's residue GEMM splits k
-    (blocks of 1536, 1024 and 40 columns in 2, 3 and 6 parts on a GB300),
-    with a fallback row and a zero column."""
-    m, n, k = 64, 2600, 5000
+    (blocks of 1536 and 1064 columns in 2 and 5 parts on a GB300), with a
+    fallback row and a zero column.  C equals the device-buffer entry's bit
+    for bit, whose sampled outputs, scales and flags are checked against the
+    oracle."""
+    m, n, k = 128, 2600, 20000
     plan = oz.oz2_plan(m, n, k, 12)
-    assert plan["host_widths"] == [1536, 1024, 40] and min(plan["host_kparts"]) > 1
+    assert plan["host_widths"] == [1536, 1064] and min(plan["host_kparts"][:2]) > 1
     A = np.array(wl.random_matrix(m, k, 1.0, 7500), order="F")
     B = np.array(wl.random_matrix(k, n, 1.0, 7600), order="F")
     A[9, :] *= 2.0 ** -300
     B[:, 2000] = 0.0
+    want = check_full_size(oz, A, B, 12, rows=np.array([0, 9, 64, 127]), cols=sample_cols(n, 30, 8))
     got = oz.oz2_dgemm_host(A, B, num_moduli=12)
-    assert_same(got, orc.oz2_dgemm(A, B, 12).C)
+    assert_same(got, want.cpu().numpy())
+    assert oz.oz2_check_device_status() == 0
+
+
+def test_operand_chunks_merge_scans(oz):
+    """A of 128 MB arrives in four column chunks.  Row 5's largest entry and
+    row 77's outlier (2^400, a fallback row) lie in later chunks, row 300
+    holds a NaN in the second; column 7 of B is 2^-300 (a fallback column).
+    C equals the device-buffer entry's bit for bit, whose flags, exponents,
+    scales and sampled outputs are checked against the oracle."""
+    m, n, k = 2048, 512, 8192
+    A = np.array(wl.random_matrix(m, k, 0.5, 7700), order="F")
+    B = np.array(wl.random_matrix(k, n, 0.5, 7800), order="F")
+    A[5, 7000] = 2.0 ** 40
+    A[77, 5000] = 2.0 ** 400
+    A[300, 3000] = np.nan
+    B[:, 7] *= 2.0 ** -300
+    rows = np.array([0, 5, 77, 1024, m - 1])  # row 300 (NaN) is compared with the device entry only
+    want = check_full_size(oz, A, B, 12, rows=rows, cols=np.unique(np.concatenate([[7], sample_cols(n, 24, 9)])))
+    got = oz.oz2_dgemm_host(A, B, num_moduli=12)
+    assert_same(got, want.cpu().numpy())
+    st = oz.oz2_get_stats()
+    assert st["fallback_rows"] == 2 and st["fallback_cols"] == 1
     assert oz.oz2_check_device_status() == 0

@@ -60,22 +60,76 @@ def test_split_invariants(oz):
     assert splits > 300
 
 
+# The host entry's block model (rates of the residue GEMM per CTA pair, of
+# the reconstruction and of the host link, with per-unit, per-block and
+# per-copy overheads), restated here to check the planner's optimisation.
+MODEL = dict(pair_flops=46e12, unit_extra=2e-6, crt_bytes=4.0e12, link=190e9, block_extra=8e-6,
+             copy_extra=5e-6)
+
+
+def model_end(widths, m, k, r, pairs):
+    """End of the last copy back for column blocks of these widths: each
+    block's compute (its residue GEMM's waves of units, then its
+    reconstruction) follows the previous block's; its copy follows both the
+    block and the previous copy."""
+    M = MODEL
+    k_pad = -(-k // 128) * 128
+    t_unit = 3 * 2 * 256 * 256 * k_pad / M["pair_flops"] + M["unit_extra"]
+    per_tile = -(-m // 256) * r
+    ce = cp = 0.0
+    for w in widths:
+        waves = -(-per_tile * -(-w // 256) // pairs)
+        ce += waves * t_unit + w * m * (2 * r + 8) / M["crt_bytes"] + M["block_extra"]
+        cp = max(ce, cp) + w * m * 8 / M["link"] + M["copy_extra"]
+    return cp
+
+
+def compositions(total, parts_max):
+    import itertools
+    for p in range(1, parts_max + 1):
+        for cuts in itertools.combinations(range(1, total), p - 1):
+            b = (0,) + cuts + (total,)
+            yield [b[i + 1] - b[i] for i in range(p)]
+
+
 def test_host_blocks(oz):
-    """oz2_dgemm_host's column blocks: the documented 4096² blocking, and over
-    seeded shapes widths that cover n, multiples of 256 but the last, which
-    is the last tile column."""
+    """oz2_dgemm_host's column blocks: the 4096³ blocking, the shape of the
+    plan at both ends of k (long k: a narrow last block, whose copy is the
+    one left exposed; short k, where the link is the bottleneck: a narrow
+    first block, which starts the copies early), and widths that cover n in
+    multiples of 256 but the last, at most 8 of them."""
     P = oz.oz2_plan(4096, 4096, 4096, 12, cta_pairs=PAIRS)
-    assert P["host_widths"] == [1280, 1280, 1280, 256]
+    assert P["host_widths"] == [2304, 768, 768, 256]
+    w = oz.oz2_plan(16384, 16384, 16384, 13, cta_pairs=PAIRS)["host_widths"]
+    assert w[-1] == 256 and w[0] > 8192
+    w = oz.oz2_plan(16384, 16384, 64, 12, cta_pairs=PAIRS)["host_widths"]
+    assert w[0] == 256 and w == sorted(w)
     assert oz.oz2_plan(300, 1000, 64, 12)["host_widths"] == [1000]  # narrow C: one block
     rng = np.random.default_rng(18)
-    for _ in range(2000):
+    for _ in range(300):
         m, n = int(rng.integers(1, 20000)), int(rng.integers(1, 40000))
         r = int(rng.integers(1, 17))
-        w = oz.oz2_plan(m, n, 1024, r, cta_pairs=PAIRS)["host_widths"]
+        w = oz.oz2_plan(m, n, int(rng.integers(1, 40000)), r, cta_pairs=PAIRS)["host_widths"]
         assert 1 <= len(w) <= 8 and sum(w) == n
-        if len(w) > 1:
-            assert all(x % 256 == 0 and x >= 768 for x in w[:-1])
-            assert w[-1] == n - 256 * (-(-n // 256) - 1)
+        assert all(x % 256 == 0 and x > 0 for x in w[:-1])
+
+
+def test_host_blocks_are_the_model_optimum(oz):
+    """For C up to 12 tile columns wide, the planner's blocks end the last
+    copy as early as the best of all partitions into at most 8 blocks of
+    whole tile columns (by exhaustion) under the same model."""
+    rng = np.random.default_rng(19)
+    for _ in range(40):
+        m = int(rng.integers(1, 20000))
+        n = int(rng.integers(257, 12 * 256 + 1))
+        k = int(rng.integers(1, 30000))
+        r = int(rng.integers(1, 17))
+        pairs = int(rng.integers(1, 80))
+        w = oz.oz2_plan(m, n, k, r, cta_pairs=pairs)["host_widths"]
+        tiles_n = -(-n // 256)
+        best = min(model_end([256 * t for t in c[:-1]] + [n - 256 * (tiles_n - c[-1])], m, k, r, pairs)
+                   for c in compositions(tiles_n, 8))
+        assert model_end(w, m, k, r, pairs) <= best * (1 + 1e-9), (m, n, k, r, pairs, w)
 
 
 def test_plan_argument_errors(oz):
