@@ -226,7 +226,7 @@ __device__ __forceinline__ double round_to_double_big(u64 hi, u64 lo, int E, boo
   return round_to_double(top, (lo << (64 - sh)) != 0, E + sh, neg);
 }
 
-// Nearest double to X·2^E for X = Hs·2^64 + L (two's complement, |X| < 2^111).
+// Nearest double to X·2^E for X = Hs·2^64 + L (two's complement, |X| < 2^127).
 // The common case (|X| ≥ 2^64, normal result) takes the leading 64 bits with
 // two funnel shifts and lets the hardware conversion round them: a sticky
 // bit for the rest is folded into bit 0, below the rounding position (bit
@@ -242,7 +242,7 @@ __device__ __forceinline__ double finish_words(long long Hs, u64 L, int E) {
   if (hi == 0) return round_to_double(lo, false, E, neg);
   const uint32_t w3 = static_cast<uint32_t>(hi >> 32), w2 = static_cast<uint32_t>(hi);
   const uint32_t w1 = static_cast<uint32_t>(lo >> 32), w0 = static_cast<uint32_t>(lo);
-  const int s = w3 ? __clz(w3) : 32 + __clz(w2);  // leading zeros of hi, 17..63
+  const int s = w3 ? __clz(w3) : 32 + __clz(w2);  // leading zeros of hi (8..63 for |X| < 2^120)
   const int e2 = E + 127 - s;                      // exponent of the leading bit of X·2^E
   if (e2 < -1022 || e2 > 1022) return round_to_double_big(hi, lo, E, neg);
   const bool ge = s >= 32;
@@ -293,6 +293,45 @@ __device__ __forceinline__ bool crt_value_w64(const int (&c)[R], int E, const Oz
   const long long zh = static_cast<long long>(yh) * mods.crt_m51h + (mid >> 32);  // ≈ X/2^51
   const long long H = (zh - static_cast<long long>(static_cast<uint32_t>(L >> 51)) + 4096) >> 13;
   out = finish_words(H, L, E);
+  return true;
+}
+
+// Fast path for r = 13 (2^112 < M < 2^121).  |X| < M/2 < 2^120, so X is
+// its own residue mod 2^128 read as a signed 128-bit word, and sums that wrap
+// around mod 2^128 suffice.  With u_k = c_k + coff_k ≥ 0, S = Σ u_k W_k ≡ X
+// (mod M); q = ⌊S/M + 1/2⌋ comes from the 32.32 fixed-point sum
+// Σ u_k F_k + 2^31 as in the five-limb path (returning false when its
+// fraction is within 2^-13 of an integer, X that close to ±M/2); and
+// X = (S − q·M) mod 2^128.  S mod 2^128 is formed from the word sums
+// A_j = Σ u_k w_kj (w_kj the 32-bit words of W_k, j = 0..2; u_k < 2^16.1, so
+// A_j < 2^52) and the top word's sum mod 2^32: four multiply-adds per
+// modulus against the five-limb path's six, and no exact S.
+template <int R>
+__device__ __forceinline__ bool crt_value_w128(const int (&c)[R], int E, const Oz2Moduli& mods, double& out) {
+  u64 a0 = 0, a1 = 0, a2 = 0;
+  uint32_t a3 = 0;
+  u64 Q = 1ull << 31;
+#pragma unroll
+  for (int k = 0; k < R; ++k) {
+    const uint32_t u = static_cast<uint32_t>(c[k] + mods.coff[k]);
+    a0 += static_cast<u64>(u) * mods.crtw[k][0];
+    a1 += static_cast<u64>(u) * mods.crtw[k][1];
+    a2 += static_cast<u64>(u) * mods.crtw[k][2];
+    a3 += u * mods.crtw[k][3];
+    Q += static_cast<u64>(u) * mods.crtf[k];
+  }
+  const uint32_t frac = static_cast<uint32_t>(Q);
+  if (frac < (1u << 19) || frac > 0xFFFFFFFFu - (1u << 19)) return false;
+  const u64 q = Q >> 32;
+  // S mod 2^128 = hi·2^64 + lo.
+  const u64 lo = a0 + (a1 << 32);
+  const u64 hi = (a1 >> 32) + a2 + (static_cast<u64>(a3) << 32) + (lo < a0 ? 1ull : 0ull);
+  // q·M mod 2^128 (q < 2^20).
+  const u64 pl = q * mods.M[0];
+  const u64 ph = q * mods.M[1] + __umul64hi(q, mods.M[0]);
+  const u64 L = lo - pl;
+  const u64 H = hi - ph - (lo < pl ? 1ull : 0ull);
+  out = finish_words(static_cast<long long>(H), L, E);
   return true;
 }
 
@@ -375,8 +414,8 @@ __device__ __forceinline__ bool y96_finish(const Y96& y, int E, const Oz2Moduli&
 constexpr long long kCrtSentinel = 0x7FF4DEAD0BADF00Dll;  // a NaN the reconstruction never produces
 
 // The reconstruction kernel's fast path by moduli count: the exact two-word
-// direct CRT for r ≤ 12 (it defers only when X lies within M/2^12 of ±M/2)
-// and the five-limb one for r ≥ 13.  (The 96-bit estimate above costs fewer
+// direct CRT for r ≤ 12 (it defers only when X lies within M/2^12 of ±M/2),
+// the 128-bit wrap-around one for r = 13 and the five-limb one for r ≥ 14.  (The 96-bit estimate above costs fewer
 // multiplies but defers small and near-midpoint outputs; measured on one
 // GB300 it was 3% slower at 4096³ and, on wide-range data with many small
 // outputs, 20% slower, so only the fused kernel, whose per-output state must
@@ -385,6 +424,8 @@ template <int R>
 __device__ __forceinline__ bool crt_fast(const int (&c)[R], int E, const Oz2Moduli& mods, double& out) {
   if constexpr (R <= 12)
     return crt_value_w64<R>(c, E, mods, out);
+  else if constexpr (R == 13)
+    return crt_value_w128<R>(c, E, mods, out);
   else
     return crt_value_fast<R>(c, E, mods, out);
 }

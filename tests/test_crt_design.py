@@ -100,3 +100,87 @@ def test_word_path_recovers_x(r):
             else:
                 assert got == x, (r, x)
     assert deferred <= 8
+
+
+def w128_constants(r):
+    """W_k = (M/m_k)·y_k, F_k = round(2^32·y_k/m_k) and coff_k = m_k·⌈2^15/m_k⌉,
+    built here from their definitions."""
+    mods = orc.moduli(r)
+    M = 1
+    for m in mods:
+        M *= m
+    out = []
+    for m in mods:
+        Mk = M // m
+        y = pow(Mk % m, -1, m)
+        out.append((m, Mk * y, ((y << 32) + m // 2) // m, m * -(-32768 // m)))
+    return M, mods, out
+
+
+def w128_path(c, r):
+    """The r = 13 fast path's word arithmetic on Python integers: word sums
+    of u_k = c_k + coff_k over W_k's 32-bit words, the 32.32 quotient sum,
+    and S - q·M mod 2^128 read as a signed word.  Returns X, or None where
+    the quotient is ambiguous."""
+    M, mods, cs = w128_constants(r)
+    m64, m32 = (1 << 64) - 1, (1 << 32) - 1
+    a = [0, 0, 0]
+    a3 = 0
+    Q = 1 << 31
+    for ck, (m, W, F, coff) in zip(c, cs):
+        u = ck + coff
+        assert 0 <= u < 2 ** 16.1
+        for j in range(3):
+            a[j] += u * ((W >> (32 * j)) & m32)
+        a3 = (a3 + u * ((W >> 96) & m32)) & m32
+        Q += u * F
+    assert max(a) < 2 ** 52 and Q < 2 ** 64
+    frac = Q & m32
+    if frac < (1 << 19) or frac > m32 - (1 << 19):
+        return None
+    q = Q >> 32
+    assert q < 2 ** 20
+    lo = (a[0] + (a[1] << 32)) & m64
+    hi = ((a[1] >> 32) + a[2] + (a3 << 32) + (1 if lo < a[0] else 0)) & m64
+    pl = (q * (M & m64)) & m64
+    ph = (q * ((M >> 64) & m64) + ((q * (M & m64)) >> 64)) & m64
+    L = (lo - pl) & m64
+    H = (hi - ph - (1 if lo < pl else 0)) & m64
+    X = (H << 64) | L
+    return X - (1 << 128) if X >> 127 else X
+
+
+def test_w128_range():
+    """r = 13 is the one count past the two-word path whose X fits a signed
+    128-bit word with room: 2^112 < M < 2^121; r = 14 does not fit."""
+    M13, _, cs = w128_constants(13)
+    assert 2 ** 112 < M13 < 2 ** 121
+    assert all(W < 2 ** 128 for _, W, _, _ in cs)
+    assert w128_constants(14)[0] > 2 ** 128
+
+
+def test_w128_path_recovers_x():
+    r = 13
+    M, mods, _ = w128_constants(r)
+    rng = random.Random(13)
+    lo, hi = -(M // 2), M - M // 2 - 1
+    xs = [0, 1, -1, lo, hi, lo + 1, hi - 1, (1 << 64), -(1 << 64), (1 << 64) - 1, -(1 << 119), (1 << 119)]
+    xs += [rng.randrange(lo, hi + 1) for _ in range(400)]
+    xs += [rng.randrange(-(1 << 70), 1 << 70) for _ in range(100)]
+    xs += [lo + rng.randrange(M >> 12) for _ in range(50)] + [hi - rng.randrange(M >> 12) for _ in range(50)]
+    deferred = 0
+    for x in xs:
+        c = [int(orc.centred(x % m, m)) for m in mods]
+        # also other int16 representatives of the same residues
+        c2 = [ck + m if ck < 0 else ck - m if ck > 0 else ck for ck, m in zip(c, mods)]
+        c3 = [ck + m * ((32767 - ck) // m) if ck < -100 else ck - m * ((ck + 32768) // m)
+              for ck, m in zip(c, mods)]  # representatives at the ends of the int16 range
+        for cc in (c, c2, c3):
+            assert all(-2 ** 15 <= v < 2 ** 15 for v in cc)
+            got = w128_path(cc, r)
+            if got is None:
+                deferred += 1
+                assert abs(x) > M // 2 - (M >> 12), x
+            else:
+                assert got == x, x
+    assert deferred <= 3 * 106  # only the 100 band samples and the ends of the range
