@@ -4,8 +4,8 @@
 // X·2^-(d_i+e_j) to FP64, including the subnormal range.
 //
 // X is computed by the direct CRT sum in fixed point (multiply-adds only):
-// an exact two-word sum for r ≤ 12, 128-bit wrap-around sums for r = 13 and
-// a five-limb sum for r ≥ 14, with
+// an exact two-word sum for r ≤ 12 and 128- and 160-bit wrap-around sums
+// for r = 13 and r ≥ 14, with
 // Garner's algorithm, the paper's method, taking over in the rare case where
 // that sum's quotient is ambiguous.  Every output equals the Garner result
 // exactly.
@@ -31,7 +31,8 @@ constexpr int kCrtFailSlots = 8;  // outputs per thread the fast path may leave 
 // Resident blocks per SM the register budget is sized for: the two-word
 // path fits 64 registers (four blocks) up to r = 12 in the FAST kernel and
 // up to r = 10 in the element-wise one; the 128-bit path (r = 13) 80 (three
-// blocks); the five-limb path (r ≥ 14) takes 128.
+// blocks); the 160-bit path (r ≥ 14) takes 128 (at 80 it spills and ran
+// 13 to 41% slower).
 template <int R, bool FAST>
 constexpr int crt_min_blocks() {
   return R <= (FAST ? 12 : 10) ? 4 : (R <= 13 ? 3 : 2);

@@ -335,6 +335,76 @@ __device__ __forceinline__ bool crt_value_w128(const int (&c)[R], int E, const O
   return true;
 }
 
+// Fast path for r = 14..16 (2^121 < M < 2^148): the same with 160-bit
+// wrap-around sums, since |X| < 2^147.  S' mod 2^160 is formed from word
+// sums over W_k's words 0..3 (below 2^53 for 16 moduli) and word 4's sum
+// mod 2^32; q (< 2^21) and its ambiguity test are the five-limb path's.
+// Five 64-bit and one 32-bit multiply-add per modulus against six 64-bit
+// ones, and the subtraction of q·M and the normalisation run on three words
+// instead of six limbs.
+template <int R>
+__device__ __forceinline__ bool crt_value_w160(const int (&c)[R], int E, const Oz2Moduli& mods, double& out) {
+  u64 a0 = 0, a1 = 0, a2 = 0, a3 = 0;
+  uint32_t a4 = 0;
+  u64 Q = 1ull << 31;
+#pragma unroll
+  for (int k = 0; k < R; ++k) {
+    const uint32_t u = static_cast<uint32_t>(c[k] + mods.coff[k]);
+    a0 += static_cast<u64>(u) * mods.crtw[k][0];
+    a1 += static_cast<u64>(u) * mods.crtw[k][1];
+    a2 += static_cast<u64>(u) * mods.crtw[k][2];
+    a3 += static_cast<u64>(u) * mods.crtw[k][3];
+    a4 += u * mods.crtw[k][4];
+    Q += static_cast<u64>(u) * mods.crtf[k];
+  }
+  const uint32_t frac = static_cast<uint32_t>(Q);
+  if (frac < (1u << 19) || frac > 0xFFFFFFFFu - (1u << 19)) return false;
+  const u64 q = Q >> 32;
+  // S' mod 2^160 = top·2^128 + mid·2^64 + lo.
+  const u64 lo = a0 + (a1 << 32);
+  const u64 s1 = (a1 >> 32) + a2 + (lo < a0 ? 1ull : 0ull);
+  const u64 mid = s1 + (a3 << 32);
+  const uint32_t top = static_cast<uint32_t>(a3 >> 32) + a4 + (mid < s1 ? 1u : 0u);
+  // q·M mod 2^160 (M's words 0..2 as 64-bit limbs, the last below 2^20).
+  const u128 p0 = static_cast<u128>(q) * mods.M[0];
+  const u128 p1 = static_cast<u128>(q) * mods.M[1] + static_cast<u64>(p0 >> 64);
+  const u64 pl = static_cast<u64>(p0), pm = static_cast<u64>(p1);
+  const uint32_t pt = static_cast<uint32_t>(static_cast<u64>(p1 >> 64) + q * mods.M[2]);
+  u64 L = lo - pl;
+  const uint32_t b0 = lo < pl ? 1u : 0u;
+  u64 Mw = mid - pm - b0;
+  const uint32_t b1 = (mid < pm || (mid == pm && b0)) ? 1u : 0u;
+  uint32_t T = top - pt - b1;
+  // Magnitude of the signed 160-bit X = T:Mw:L.
+  const bool neg = (T >> 31) != 0;
+  if (neg) {
+    L = 0ull - L;
+    const uint32_t c0 = L == 0 ? 1u : 0u;
+    Mw = ~Mw + c0;
+    T = ~T + ((c0 && Mw == 0) ? 1u : 0u);
+  }
+  // Leading 64 bits and a sticky bit for the rest.
+  u64 top64;
+  bool sticky;
+  if (T != 0) {
+    const int z = __clz(T);                      // 0..31
+    const int sh = 32 - z;                       // bits of T
+    top64 = (static_cast<u64>(T) << (64 - sh)) | (Mw >> sh);
+    sticky = (Mw << (64 - sh)) != 0 || L != 0;
+    E += 64 + sh;
+  } else if (Mw != 0) {
+    const int sh = 64 - __clzll(static_cast<long long>(Mw));  // 1..64
+    top64 = sh == 64 ? Mw : (Mw << (64 - sh)) | (L >> sh);
+    sticky = sh == 64 ? L != 0 : (L << (64 - sh)) != 0;
+    E += sh;
+  } else {
+    top64 = L;
+    sticky = false;
+  }
+  out = round_to_double(top64, sticky, E, neg);
+  return true;
+}
+
 // 96-bit estimate for r = 11, 12 (2^102 < M < 2^112): one fixed-point sum.
 // With F_k = round(2^96·y_k/m_k), Y = Σ c_k F_k mod 2^96 read as a signed
 // word is 2^96·X/M + D with |D| ≤ Σ|c_k|/2, as long as that stays inside
@@ -415,7 +485,8 @@ constexpr long long kCrtSentinel = 0x7FF4DEAD0BADF00Dll;  // a NaN the reconstru
 
 // The reconstruction kernel's fast path by moduli count: the exact two-word
 // direct CRT for r ≤ 12 (it defers only when X lies within M/2^12 of ±M/2),
-// the 128-bit wrap-around one for r = 13 and the five-limb one for r ≥ 14.  (The 96-bit estimate above costs fewer
+// and the 128-bit and 160-bit wrap-around ones for r = 13 and r ≥ 14.
+// (The 96-bit estimate above costs fewer
 // multiplies but defers small and near-midpoint outputs; measured on one
 // GB300 it was 3% slower at 4096³ and, on wide-range data with many small
 // outputs, 20% slower, so only the fused kernel, whose per-output state must
@@ -427,7 +498,7 @@ __device__ __forceinline__ bool crt_fast(const int (&c)[R], int E, const Oz2Modu
   else if constexpr (R == 13)
     return crt_value_w128<R>(c, E, mods, out);
   else
-    return crt_value_fast<R>(c, E, mods, out);
+    return crt_value_w160<R>(c, E, mods, out);
 }
 
 // The exact paths, for outputs the fast path leaves: the two-word direct CRT

@@ -184,3 +184,68 @@ def test_w128_path_recovers_x():
             else:
                 assert got == x, x
     assert deferred <= 3 * 106  # only the 100 band samples and the ends of the range
+
+
+def w160_path(c, r):
+    """The r = 14..16 fast path's word arithmetic on Python integers: word
+    sums of u_k over W_k's words 0..3 and word 4 mod 2^32, the 32.32 quotient
+    sum, S' - q·M mod 2^160 read as a signed word.  Returns X, or None where
+    the quotient is ambiguous."""
+    M, mods, cs = w128_constants(r)
+    m64, m32 = (1 << 64) - 1, (1 << 32) - 1
+    a = [0, 0, 0, 0]
+    a4 = 0
+    Q = 1 << 31
+    for ck, (m, W, F, coff) in zip(c, cs):
+        u = ck + coff
+        for j in range(4):
+            a[j] += u * ((W >> (32 * j)) & m32)
+        a4 = (a4 + u * ((W >> 128) & m32)) & m32
+        Q += u * F
+    assert max(a) < 2 ** 53 and Q < 2 ** 64
+    frac = Q & m32
+    if frac < (1 << 19) or frac > m32 - (1 << 19):
+        return None
+    q = Q >> 32
+    assert q < 2 ** 21
+    lo = (a[0] + (a[1] << 32)) & m64
+    s1 = (a[1] >> 32) + a[2] + (1 if lo < a[0] else 0)
+    assert s1 < 2 ** 64
+    mid = (s1 + (a[3] << 32)) & m64
+    top = ((a[3] >> 32) + a4 + (1 if mid < s1 else 0)) & m32
+    P = q * M
+    X = ((top << 128) | (mid << 64) | lo) - P
+    X &= (1 << 160) - 1
+    return X - (1 << 160) if X >> 159 else X
+
+
+def test_w160_range():
+    """r = 14..16 fit a signed 160-bit word: M < 2^148, W_k < 2^160, and the
+    top word of M (bits 128 and up) is below 2^20."""
+    for r in (14, 15, 16):
+        M, _, cs = w128_constants(r)
+        assert 2 ** 121 < M < 2 ** 148
+        assert all(W < 2 ** 160 for _, W, _, _ in cs)
+        assert (M >> 128) < 2 ** 20
+
+
+@pytest.mark.parametrize("r", [14, 16])
+def test_w160_path_recovers_x(r):
+    M, mods, _ = w128_constants(r)
+    rng = random.Random(r)
+    lo, hi = -(M // 2), M - M // 2 - 1
+    xs = [0, 1, -1, lo, hi, lo + 1, hi - 1, 1 << 64, -(1 << 64), 1 << 128, -(1 << 128), (1 << 128) - 1]
+    xs += [rng.randrange(lo, hi + 1) for _ in range(300)]
+    xs += [rng.randrange(-(1 << 100), 1 << 100) for _ in range(60)]
+    xs += [lo + rng.randrange(M >> 12) for _ in range(30)] + [hi - rng.randrange(M >> 12) for _ in range(30)]
+    for x in xs:
+        c = [int(orc.centred(x % m, m)) for m in mods]
+        c2 = [ck + m if ck < 0 else ck - m if ck > 0 else ck for ck, m in zip(c, mods)]
+        c3 = [ck + m * ((32767 - ck) // m) if ck < -100 else ck - m * ((ck + 32768) // m)
+              for ck, m in zip(c, mods)]
+        for cc in (c, c2, c3):
+            got = w160_path(cc, r)
+            if got is None:
+                assert abs(x) > M // 2 - (M >> 12), x
+            else:
+                assert got == x, x

@@ -135,12 +135,15 @@ def test_column_blocks_with_split_k(oz):
     assert oz.oz2_check_device_status() == 0
 
 
-def test_operand_chunks_merge_scans(oz):
-    """A of 128 MB arrives in four column chunks.  Row 5's largest entry and
-    row 77's outlier (2^400, a fallback row) lie in later chunks, row 300
-    holds a NaN in the second; column 7 of B is 2^-300 (a fallback column).
-    C equals the device-buffer entry's bit for bit, whose flags, exponents,
-    scales and sampled outputs are checked against the oracle."""
+@pytest.mark.parametrize("pad", [0, 3])
+def test_operand_chunks_merge_scans(oz, pad):
+    """A of 128 MB arrives in four column chunks (pitched copies when its
+    leading dimension is m + pad).  Row 5's largest entry and row 77's
+    outlier (2^400, a fallback row) lie in later chunks, row 300 holds a NaN
+    in the second; column 7 of B is 2^-300 (a fallback column).  C equals
+    the device-buffer entry's bit for bit, whose flags, exponents, scales
+    and sampled outputs are checked against the oracle."""
+    import torch
     m, n, k = 2048, 512, 8192
     A = np.array(wl.random_matrix(m, k, 0.5, 7700), order="F")
     B = np.array(wl.random_matrix(k, n, 0.5, 7800), order="F")
@@ -150,7 +153,12 @@ def test_operand_chunks_merge_scans(oz):
     B[:, 7] *= 2.0 ** -300
     rows = np.array([0, 5, 77, 1024, m - 1])  # row 300 (NaN) is compared with the device entry only
     want = check_full_size(oz, A, B, 12, rows=rows, cols=np.unique(np.concatenate([[7], sample_cols(n, 24, 9)])))
-    got = oz.oz2_dgemm_host(A, B, num_moduli=12)
+    hA = A
+    if pad:
+        hA = torch.full((k, m + pad), 5.0, dtype=torch.float64, pin_memory=True).t()[:m]
+        hA.copy_(torch.from_numpy(A))
+        assert hA.stride() == (1, m + pad)
+    got = oz.oz2_dgemm_host(hA, B, num_moduli=12)
     assert_same(got, want.cpu().numpy())
     st = oz.oz2_get_stats()
     assert st["fallback_rows"] == 2 and st["fallback_cols"] == 1
