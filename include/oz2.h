@@ -234,6 +234,13 @@ int oz2_workspace_layout(int64_t m, int64_t n, int64_t k, int num_moduli,
  *                 the copies dominate, a narrow first one (the copies start
  *                 early).  Identical shapes reuse the last plan.
  *   host_kparts   the residue GEMM's kparts for each block.
+ *   mag_kparts    parts of k of the "+1" magnitude GEMM (1: no split).
+ *                 When its 256×256 tiles fill less than half a wave (a
+ *                 small C with a long k), each tile runs in up to 64 parts
+ *                 of at least 512 k-entries; the parts add their FP32 sums
+ *                 (exact: integers in units of 2^-2c below 2^24) into an
+ *                 m×n buffer in the then unused digit-plane region, and a
+ *                 row-maximum kernel follows (one launch more).
  * Returns OZ2_OK, OZ2_ERR_INVALID_ARG (null out, negative sizes,
  * cta_pairs < 1) or OZ2_ERR_UNSUPPORTED_R. */
 typedef struct {
@@ -241,6 +248,7 @@ typedef struct {
   int32_t host_blocks;
   int64_t host_widths[8];
   int64_t host_kparts[8];
+  int64_t mag_kparts;
 } oz2_plan_info;
 int oz2_plan(int64_t m, int64_t n, int64_t k, int num_moduli, int cta_pairs, oz2_plan_info* out);
 

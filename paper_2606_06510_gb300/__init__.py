@@ -54,7 +54,8 @@ class oz2_ws_layout(ctypes.Structure):
 
 class oz2_plan_info(ctypes.Structure):
     _fields_ = [("kparts", ctypes.c_int64), ("host_blocks", ctypes.c_int32),
-                ("host_widths", ctypes.c_int64 * 8), ("host_kparts", ctypes.c_int64 * 8)]
+                ("host_widths", ctypes.c_int64 * 8), ("host_kparts", ctypes.c_int64 * 8),
+                ("mag_kparts", ctypes.c_int64)]
 
 
 _I64, _P, _I, _U, _SZ = ctypes.c_int64, ctypes.c_void_p, ctypes.c_int, ctypes.c_uint, ctypes.c_size_t
@@ -185,12 +186,14 @@ def oz2_workspace_layout(m: int, n: int, k: int, num_moduli: int) -> dict:
 
 def oz2_plan(m: int, n: int, k: int, num_moduli: int = 12, cta_pairs: int = 76) -> dict:
     """How the library runs an m×n×k problem on cta_pairs CTA pairs (host
-    arithmetic only): the residue GEMM's parts of k, and the column blocks
-    of oz2_dgemm_host with each block's parts of k."""
+    arithmetic only): the residue GEMM's parts of k, the column blocks of
+    oz2_dgemm_host with each block's parts of k, and the "+1" magnitude
+    GEMM's parts of k."""
     P = oz2_plan_info()
     _check(lib().oz2_plan(m, n, k, num_moduli, cta_pairs, ctypes.byref(P)), "oz2_plan")
     nb = P.host_blocks
-    return {"kparts": P.kparts, "host_widths": list(P.host_widths[:nb]), "host_kparts": list(P.host_kparts[:nb])}
+    return {"kparts": P.kparts, "host_widths": list(P.host_widths[:nb]), "host_kparts": list(P.host_kparts[:nb]),
+            "mag_kparts": P.mag_kparts}
 
 
 def oz2_plane_layout(num_moduli: int):

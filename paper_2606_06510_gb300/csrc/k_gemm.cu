@@ -54,6 +54,8 @@ struct EpiCtx {
   float* urow;
   Oz2Device* dev;
   int64_t m, n, ldr;
+  float* upart;   // magnitude GEMM split along k: U (m×n row-major, ld = ldu) summed over the parts
+  int64_t ldu;    // a multiple of 4: 16-byte rows
 };
 
 // Units: (modulus, part of the k-blocks, tile).  With kparts > 1 (split K)
@@ -76,14 +78,16 @@ struct Unit {
 // Unit u (grouped raster of kGroupM tile rows).  Modulus block j of the
 // units is modulus nsq + j for the nheavy nonsquare moduli, then modulus
 // j - nheavy for the squares; within a modulus the parts come in order.
-// The magnitude GEMM (MODE 1) has one modulus and never splits K.
+// The magnitude GEMM (MODE 1) has one modulus; its parts of k (when it is
+// split) come in order, each over all tiles.
 template <int MODE>
 __device__ __forceinline__ Unit unit_at(int64_t u, const UnitMap& um) {
   Unit x;
   int64_t t = u;
   if (MODE == 1) {
     x.i = 0;
-    x.part = 0;
+    x.part = static_cast<int>(u / um.ntiles);
+    t = u - static_cast<int64_t>(x.part) * um.ntiles;
   } else {
     const int64_t per_mod = um.ntiles * um.kparts;
     const int j = static_cast<int>(u / per_mod);
@@ -99,13 +103,8 @@ __device__ __forceinline__ Unit unit_at(int64_t u, const UnitMap& um) {
   const int64_t local = t - g * per_group;
   x.tm = first + local % gm;
   x.tn = local / gm;
-  if (MODE == 1) {
-    x.k_lo = 0;
-    x.k_hi = um.ksteps;
-  } else {
-    x.k_lo = static_cast<int64_t>(x.part) * um.kpart_steps;
-    x.k_hi = um.ksteps - x.k_lo < um.kpart_steps ? um.ksteps : x.k_lo + um.kpart_steps;
-  }
+  x.k_lo = static_cast<int64_t>(x.part) * um.kpart_steps;
+  x.k_hi = um.ksteps - x.k_lo < um.kpart_steps ? um.ksteps : x.k_lo + um.kpart_steps;
   return x;
 }
 
@@ -121,7 +120,7 @@ __device__ __forceinline__ int planes_of(const Oz2Moduli& mods, int i) {
 }
 template <int MODE>
 __device__ __forceinline__ int64_t slab_steps_of(const Oz2Moduli& mods, int i, int64_t ksteps) {
-  if (MODE == 1) return ksteps;
+  if (MODE == 1) return ksteps;  // the magnitude sums stay below 2^24 units over all of k
   return (mods.sq_base[i] ? kKSlabSquare : kKSlabMerged) / kBK;
 }
 
@@ -358,7 +357,23 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
             __syncwarp();
             if (lane == 0) mbar_arrive_remote_relaxed(acc_empty_leader);
           }
-          if (MODE == 1) {
+          if (MODE == 1 && ctx.upart) {  // a part of k: add this tile's partial sums into U
+            const int64_t cc = col0 + c;
+            if (row < ctx.m) {
+              float* dst = ctx.upart + row * ctx.ldu + cc;  // 16-byte aligned: ldu and cc multiples of 4
+              if (cc + 16 <= ctx.n) {
+#pragma unroll
+                for (int j = 0; j < 16; j += 4)
+                  atomicAdd(reinterpret_cast<float4*>(dst + j),
+                            make_float4(__uint_as_float(v0[j]), __uint_as_float(v0[j + 1]), __uint_as_float(v0[j + 2]),
+                                        __uint_as_float(v0[j + 3])));
+              } else {
+#pragma unroll
+                for (int j = 0; j < 16; ++j)
+                  if (cc + j < ctx.n) atomicAdd(dst + j, __uint_as_float(v0[j]));
+              }
+            }
+          } else if (MODE == 1) {
 #pragma unroll
             for (int j = 0; j < 16; ++j) rowmax = fmaxf(rowmax, __uint_as_float(v0[j]));
           } else if (carry) {  // every lane: tcgen05.st is warp-collective
@@ -425,7 +440,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         }
         accph ^= 1;
       }
-      if (MODE == 1 && ok) {
+      if (MODE == 1 && ok && !ctx.upart) {
         // rows past m hold zeros (TMA fills out-of-range rows with 0)
         if (row < ctx.m) atomicMax(reinterpret_cast<int*>(ctx.urow) + row, __float_as_int(rowmax));
         const int wm = __reduce_max_sync(0xffffffffu, __float_as_int(rowmax));
@@ -702,6 +717,49 @@ int64_t residue_gemm_kparts(int64_t m, int64_t n, int64_t k_pad, int r, int nsq,
 
 static size_t gemm_smem_bytes() { return 1024 + static_cast<size_t>(kStages) * kStageBytes + 8 * (2 * kStages + 3); }
 
+// The magnitude GEMM split along k: each part adds its tiles' partial sums
+// into U with 16-byte vector atomics (every partial sum is an integer number
+// of units 2^-2c below 2^24, like the whole sum, so FP32 adds them exactly in
+// any order), and this kernel then takes each row's maximum, as the unsplit
+// epilogue does: a warp per row of the row-major U.
+constexpr int kRowMaxThreads = 256;
+__global__ void __launch_bounds__(kRowMaxThreads) plus_one_rowmax_kernel(const float* __restrict__ U, int64_t m,
+                                                                         int64_t n, int64_t ldu,
+                                                                         float* __restrict__ urow, Oz2Device* dev) {
+  const int lane = threadIdx.x & 31;
+  const int64_t row = static_cast<int64_t>(blockIdx.x) * (kRowMaxThreads / 32) + (threadIdx.x >> 5);
+  if (row >= m) return;  // whole warps
+  float mx = 0.f;
+  const float* p = U + row * ldu;
+  for (int64_t col = lane; col < n; col += 32) mx = fmaxf(mx, __ldg(p + col));
+  const int wm = __reduce_max_sync(0xffffffffu, __float_as_int(mx));  // nonnegative floats order as their bits
+  if (lane == 0) {
+    atomicMax(reinterpret_cast<int*>(urow) + row, wm);
+    atomicMax(&dev->u_max_bits, wm);
+  }
+}
+
+// Parts of k for the magnitude GEMM: its 256×256 tiles fill fewer than half
+// a wave of the CTA pairs only for a small C with a long k; then each tile
+// runs in as many parts as the pairs allow (at most 64, each at least
+// kMinPartSteps k-blocks), and U's partial sums go through scratch.
+static int64_t magnitude_ldu(int64_t n) { return (n + 3) / 4 * 4; }
+
+static int64_t magnitude_kparts(int64_t ntiles, int64_t ksteps, int64_t pairs, int64_t m, int64_t n,
+                                size_t scratch_bytes) {
+  if (2 * ntiles >= pairs || scratch_bytes < static_cast<size_t>(m) * magnitude_ldu(n) * sizeof(float)) return 1;
+  int64_t p = std::min<int64_t>({64, pairs / ntiles, ksteps / kMinPartSteps});
+  if (p < 2) return 1;
+  const int64_t s = (ksteps + p - 1) / p;
+  return (ksteps + s - 1) / s;  // no empty part
+}
+
+int64_t magnitude_gemm_kparts(int64_t m, int64_t n, int64_t k_pad, size_t scratch_bytes, int64_t pairs) {
+  if (m <= 0 || n <= 0 || k_pad <= 0 || pairs < 1) return 1;
+  const int64_t ntiles = ((m + kTileM - 1) / kTileM) * ((n + kTileN - 1) / kTileN);
+  return magnitude_kparts(ntiles, k_pad / kBK, pairs, m, n, scratch_bytes);
+}
+
 // mode: 0 residues (tensor cores), 1 magnitude (tensor cores),
 //       2 residues (SIMT reference), 3 magnitude (SIMT reference).
 cudaError_t launch_plane_gemm(int64_t m, int64_t n, int64_t k_pad, const Oz2Moduli& mods,
@@ -709,7 +767,7 @@ cudaError_t launch_plane_gemm(int64_t m, int64_t n, int64_t k_pad, const Oz2Modu
                               int16_t* residues, int64_t ldr, float* urow, Oz2Device* dev, cudaStream_t st,
                               int16_t* partials, size_t partial_bytes) {
   if (m == 0 || n == 0) return cudaSuccess;
-  EpiCtx ctx{residues, urow, dev, m, n, ldr};
+  EpiCtx ctx{residues, urow, dev, m, n, ldr, nullptr, 0};
   if (mode >= 2) {
     dim3 g(static_cast<unsigned>((m + 127) / 128), static_cast<unsigned>(n));
     count_launch();
@@ -770,10 +828,29 @@ cudaError_t launch_plane_gemm(int64_t m, int64_t n, int64_t k_pad, const Oz2Modu
     um.nunits *= um.kparts;
     if (um.kparts > 1) ctx.res = partials;
   }
+  // The magnitude GEMM of a small C with a long k: parts of k, with U's
+  // partial sums in the scratch (`partials`, 16-byte aligned).
+  if (mode == 1 && partials && reinterpret_cast<uintptr_t>(partials) % 16 == 0) {
+    um.kparts = magnitude_kparts(um.ntiles, um.ksteps, pairs, m, n, partial_bytes);
+    um.kpart_steps = (um.ksteps + um.kparts - 1) / um.kparts;
+    um.nunits *= um.kparts;
+    if (um.kparts > 1) {
+      ctx.upart = reinterpret_cast<float*>(partials);
+      ctx.ldu = magnitude_ldu(n);
+      err = cudaMemsetAsync(ctx.upart, 0, static_cast<size_t>(m) * ctx.ldu * sizeof(float), st);
+      if (err != cudaSuccess) return err;
+    }
+  }
   pairs = std::max<int64_t>(1, std::min<int64_t>(pairs, um.nunits));
   count_launch();
   kern<<<static_cast<unsigned>(2 * pairs), kGemmThreads, smem, st>>>(ta, tb, mods, k_pad, um, ctx);
-  if (um.kparts > 1) {
+  if (ctx.upart) {
+    count_launch();
+    constexpr int64_t rows_per_block = kRowMaxThreads / 32;
+    plus_one_rowmax_kernel<<<static_cast<unsigned>((m + rows_per_block - 1) / rows_per_block), kRowMaxThreads, 0,
+                             st>>>(ctx.upart, m, n, ctx.ldu, urow, dev);
+  }
+  if (mode == 0 && um.kparts > 1) {  // the residue GEMM's parts, folded into C^(i)
     const int64_t row_threads = (m + 7) / 8;
     dim3 g(static_cast<unsigned>((row_threads + kFoldThreads - 1) / kFoldThreads),
            static_cast<unsigned>(std::min<int64_t>(n, 32768)), static_cast<unsigned>(mods.r));

@@ -617,8 +617,11 @@ static int run_stages(int64_t m, int64_t n, int64_t k, const double* A, int64_t 
     if (err == cudaSuccess)
       err = launch_magnitude_planes(m, in ? 0 : n, k, A, lda, B, ldb, ra, cb, rf, cf, mag_a, mag_b, s);
     mark(2);
+    // The digit-plane and residue regions are not yet in use: the scratch
+    // for the magnitude GEMM's partial sums when it splits k.
     if (err == cudaSuccess)
-      err = launch_plane_gemm(m, n, L.k_pad, mods, mag_a, mag_b, simt ? 3 : 1, nullptr, 0, urow, ds->status, s);
+      err = launch_plane_gemm(m, n, L.k_pad, mods, mag_a, mag_b, simt ? 3 : 1, nullptr, 0, urow, ds->status, s,
+                              reinterpret_cast<int16_t*>(pa), L.total - L.planes_a);
     mark(3);
   } else {
     mark(2);
@@ -822,6 +825,7 @@ int oz2_plan(int64_t m, int64_t n, int64_t k, int num_moduli, int cta_pairs, oz2
                                L.planes_a - L.mag_a, cta_pairs);
   };
   out->kparts = kparts(n);
+  out->mag_kparts = m > 0 && n > 0 && k > 0 ? magnitude_gemm_kparts(m, n, L.k_pad, L.total - L.planes_a, cta_pairs) : 1;
   const ColumnBlocks b = host_column_blocks(m, n, num_moduli, k, cta_pairs);
   out->host_blocks = b.count;
   for (int i = 0; i < b.count; ++i) {

@@ -520,8 +520,11 @@ cudaError_t launch_deconstruct(int64_t m, int64_t n, int64_t k, const Oz2Moduli&
 // Host-only arithmetic.
 int64_t residue_gemm_kparts(int64_t m, int64_t n, int64_t k_pad, int r, int nsq, int64_t ldr, size_t partial_bytes,
                             int64_t pairs);
+int64_t magnitude_gemm_kparts(int64_t m, int64_t n, int64_t k_pad, size_t scratch_bytes, int64_t pairs);
 // `partials` (16-byte aligned, `partial_bytes` long, or null) is scratch the
-// residue GEMM may split K into; it must not overlap the operands or C^(i).
+// residue GEMM may split K into (the parts' residues), and the magnitude GEMM
+// too (the m×n FP32 sums of its parts); it must not overlap the operands,
+// C^(i) or urow.
 cudaError_t launch_plane_gemm(int64_t m, int64_t n, int64_t k_pad, const Oz2Moduli& mods,
                               const uint8_t* planes_a, const uint8_t* planes_b, int mode,
                               int16_t* residues, int64_t ldr, float* urow, Oz2Device* dev, cudaStream_t st,

@@ -4,7 +4,9 @@ A problem with few output tiles and a long k fills few waves of the CTA
 pairs, so the residue GEMM runs each unit's k-blocks in parts and sums the
 parts' residues mod m (Eq. modgemm is a sum over k).  Each case checks the
 scales, every residue matrix C^(i) and C against the oracle, and that the
-call did split: it launches one kernel more (the fold) than an unsplit call.
+call did split: it launches one kernel more (the fold) than an unsplit call,
+besides the row-maximum kernel of a split "+1" magnitude GEMM where the
+plan reports one (mag_kparts).
 """
 import numpy as np
 import pytest
@@ -17,13 +19,14 @@ pytestmark = pytest.mark.gpu
 
 
 
-def unsplit_launches(m):
-    """Kernels of an unsplit call: prepare, 2 scan (A and B in one launch,
-    then the flags), magnitude, "+1", scales, deconstruct, GEMM, CRT, 2
-    fallback.  (C here has ld = m: for even m the CRT takes every row in
-    pairs, for odd m it runs the element-wise instance alone, so it is one
-    launch either way.)"""
-    return 11
+def unsplit_launches(oz, m, n, k, r):
+    """Kernels of a call whose residue GEMM does not split: prepare, 2 scan
+    (A and B in one launch, then the flags), magnitude, "+1", scales,
+    deconstruct, GEMM, CRT, 2 fallback, and the row maxima of a split "+1"
+    GEMM.  (C here has ld = m: for even m the CRT takes every row in pairs,
+    for odd m it runs the element-wise instance alone, so it is one launch
+    either way.)"""
+    return 11 + (oz.oz2_plan(m, n, k, r, 76)["mag_kparts"] > 1)
 
 
 @pytest.fixture(scope="module")
@@ -54,7 +57,7 @@ def run_counted(oz, A, B, r):
 def check(oz, A, B, r, split):
     want = orc.oz2_dgemm(A, B, r)
     C, v, launches = run_counted(oz, A, B, r)
-    assert launches == unsplit_launches(A.shape[0]) + (1 if split else 0)
+    assert launches == unsplit_launches(oz, A.shape[0], B.shape[1], A.shape[1], r) + (1 if split else 0)
     assert np.array_equal(v["d"], want.d) and np.array_equal(v["e"], want.e)
     assert np.array_equal(v["residues"], want.residues)
     same = (C == want.C) | (np.isnan(C) & np.isnan(want.C))
@@ -104,7 +107,8 @@ def test_many_tiles_do_not_split(oz):
     A = np.array(wl.random_matrix(m, k, 0.5, 9950), order="F")
     B = np.array(wl.random_matrix(k, n, 0.5, 9951), order="F")
     C, _, launches = run_counted(oz, A, B, 12)
-    assert launches == unsplit_launches(m)
+    assert oz.oz2_plan(m, n, k, 12, 76)["kparts"] == 1
+    assert launches == unsplit_launches(oz, m, n, k, 12)
     rows = np.arange(0, m, 97)
     want = orc.oz2_dgemm(A, B, 12, rows=rows)
     assert np.array_equal(C[rows], want.C)

@@ -132,6 +132,33 @@ def test_host_blocks_are_the_model_optimum(oz):
         assert model_end(w, m, k, r, pairs) <= best * (1 + 1e-9), (m, n, k, r, pairs, w)
 
 
+def test_magnitude_gemm_split(oz):
+    """The "+1" GEMM splits k only when its 256×256 tiles fill less than half
+    a wave of the CTA pairs: none at 4096³; 4 parts for 16 tiles at
+    k = 65536 (64 units on 76 pairs); 64 for a single tile; none when k is
+    too short for two parts of 512 entries or the planes' scratch cannot
+    hold m×n FP32 sums."""
+    assert oz.oz2_plan(4096, 4096, 4096, 12, cta_pairs=PAIRS)["mag_kparts"] == 1
+    assert oz.oz2_plan(1024, 1024, 65536, 12, cta_pairs=PAIRS)["mag_kparts"] == 4
+    assert oz.oz2_plan(256, 256, 65536, 12, cta_pairs=PAIRS)["mag_kparts"] == 64
+    assert oz.oz2_plan(1536, 1280, 1536, 12, cta_pairs=PAIRS)["mag_kparts"] == 2   # 30 tiles
+    assert oz.oz2_plan(1024, 1024, 1000, 12, cta_pairs=PAIRS)["mag_kparts"] == 2   # 8 k-blocks: 2 parts of 4
+    assert oz.oz2_plan(256, 256, 512, 12, cta_pairs=PAIRS)["mag_kparts"] == 1      # 4 k-blocks: one part
+    rng = np.random.default_rng(20)
+    for _ in range(500):
+        m, n, k = int(rng.integers(1, 6000)), int(rng.integers(1, 6000)), int(rng.integers(1, 200000))
+        pairs = int(rng.integers(1, 80))
+        p = oz.oz2_plan(m, n, k, 12, cta_pairs=pairs)["mag_kparts"]
+        t = tiles(m, n)
+        ksteps = -(-k // 128)
+        if p > 1:
+            assert 2 * t < pairs and p <= 64 and p * t <= pairs
+            s = -(-ksteps // p)
+            assert s >= 4 and (p - 1) * s < ksteps         # parts of at least 4 k-blocks, none empty
+        else:
+            assert 2 * t >= pairs or min(64, pairs // t, ksteps // 4) < 2
+
+
 def test_plan_argument_errors(oz):
     with pytest.raises(oz.Oz2Error):
         oz.oz2_plan(8, 8, 8, 12, cta_pairs=0)

@@ -90,7 +90,8 @@ def test_matches_the_oracle(env):
 def test_split_k_in_the_scratch_then_an_unsplit_call(env, shape, r, parts):
     """A small C with a long k: the residue GEMM splits k and keeps the
     parts' residues in the scratch array's magnitude-plane region.  The
-    split call (one launch more than an unsplit one: the fold) must match
+    split call (two launches more than an unsplit one: the fold, and the row
+    maxima of the "+1" GEMM, which splits k as well) must match
     oz2_dgemm bit for bit, and an unsplit call right after it must too."""
     oz, _, _ = env
     m, n, k = shape
@@ -98,13 +99,15 @@ def test_split_k_in_the_scratch_then_an_unsplit_call(env, shape, r, parts):
     assert oz.oz2_plan(m, n, k, r, 76)["kparts"] == parts
     A = to_dev(wl.random_matrix(m, k, 1.0, 5151 + r))
     B = to_dev(wl.random_matrix(k, n, 1.0, 5252 + r))
+    assert oz.oz2_plan(m, n, k, r, 76)["mag_kparts"] > 1  # the "+1" GEMM splits k too
     oz.oz2_get_stats()                      # resets the launch counter
     got = call_noalloc(env, A, B, r)
-    assert oz.oz2_get_stats()["kernel_launches"] == 12
+    assert oz.oz2_get_stats()["kernel_launches"] == 13
     want = oz.oz2_dgemm(A, B, num_moduli=r).cpu().numpy()
     assert np.array_equal(got, want)
     A2 = to_dev(wl.random_matrix(96, 300, 0.5, 5353 + r))
     B2 = to_dev(wl.random_matrix(300, 80, 0.5, 5454 + r))
+    assert oz.oz2_plan(96, 80, 300, r, 76)["mag_kparts"] == 1
     oz.oz2_get_stats()
     got2 = call_noalloc(env, A2, B2, r)
     assert oz.oz2_get_stats()["kernel_launches"] == 11
