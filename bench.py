@@ -51,8 +51,8 @@ GEMM_SOURCES = [os.path.join(ROOT, "paper_2606_06510_gb300", "csrc", f)
 # DRAM read+write bytes of one residue-GEMM launch at 4096^3, r = 12, from
 # one ncu capture of that launch; reported only while the kernel's sources
 # are the ones the counters were taken on (SHA-256 over them in order).
-GEMM_TRAFFIC = {"workload": "dgemm_4096", "num_moduli": 12, "bytes": 2.1118e9,
-                "sha256": "7cb736dacb1d935d03d29c2ca93143c1b11c437fa7f443437f405cdd1b4c0d3b"}
+GEMM_TRAFFIC = {"workload": "dgemm_4096", "num_moduli": 12, "bytes": 2.1487e9,
+                "sha256": "dadebac1907b06dbb6c73c9bce18cadbbb863c1d5620e01e75330c2135c40d1e"}
 
 
 def gemm_traffic(w, r):
@@ -68,6 +68,24 @@ def gemm_traffic(w, r):
     if sha == t["sha256"] and w.name == t["workload"] and r == t["num_moduli"]:
         return t["bytes"]
     return None
+
+
+def host_link_rates(hA, dA, hC, dC, reps=3):
+    """This box's pinned host link, for reading the end-to-end figure: one
+    operand in (A) and C out as plain stream copies, CUDA-event timed."""
+    import torch
+    out = {}
+    for name, dst, src in (("h2d", dA, hA), ("d2h", hC, dC)):
+        dst.copy_(src, non_blocking=True)
+        torch.cuda.synchronize()
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t0.record()
+        for _ in range(reps):
+            dst.copy_(src, non_blocking=True)
+        t1.record()
+        torch.cuda.synchronize()
+        out[name] = round(reps * src.numel() * src.element_size() / (t0.elapsed_time(t1) * 1e6), 1)
+    return out
 
 
 def parse():
@@ -470,7 +488,8 @@ def run_oz2(args):
     e2e_s = max_over_ranks(e2e_s, world)
     e2e = {"value": round(world * w.flops / e2e_s / 1e12, 3), "unit": "TFLOPS",
            "h2d_bytes_per_step": in_bytes, "d2h_bytes_per_step": 8 * w.m * w.n,
-           "api": "oz2_dgemm_host (pinned host buffers)"}
+           "api": "oz2_dgemm_host (pinned host buffers)", "ms_per_step": round(e2e_s * 1e3, 4),
+           "host_link_gbs": host_link_rates(hA, dA, hC, dC)}
 
     extra = {}
     if rank == 0:
