@@ -125,8 +125,10 @@ __device__ __forceinline__ int64_t slab_steps_of(const Oz2Moduli& mods, int i, i
 }
 
 // MODE 0: residue planes (all moduli); MODE 1: magnitude planes ("+1" pass).
-// SHORT1: the instance for k ≤ 128 (one k-block, so one short slab for every
-// modulus), whose epilogue takes the single-correction reduction.
+// SHORT1, for MODE 0: the instance for k ≤ 128 (one k-block, so one short
+// slab for every modulus), whose epilogue takes the single-correction
+// reduction; for MODE 1: the instance whose tiles run in parts of k and add
+// their partial sums into U (EpiCtx::upart) instead of taking row maxima.
 template <int MODE, bool SHORT1 = false>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     plane_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
@@ -357,7 +359,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
             __syncwarp();
             if (lane == 0) mbar_arrive_remote_relaxed(acc_empty_leader);
           }
-          if (MODE == 1 && ctx.upart) {  // a part of k: add this tile's partial sums into U
+          if (MODE == 1 && SHORT1) {  // a part of k: add this tile's partial sums into U
             const int64_t cc = col0 + c;
             if (row < ctx.m) {
               float* dst = ctx.upart + row * ctx.ldu + cc;  // 16-byte aligned: ldu and cc multiples of 4
@@ -440,7 +442,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         }
         accph ^= 1;
       }
-      if (MODE == 1 && ok && !ctx.upart) {
+      if (MODE == 1 && !SHORT1 && ok) {
         // rows past m hold zeros (TMA fills out-of-range rows with 0)
         if (row < ctx.m) atomicMax(reinterpret_cast<int*>(ctx.urow) + row, __float_as_int(rowmax));
         const int wm = __reduce_max_sync(0xffffffffu, __float_as_int(rowmax));
@@ -835,6 +837,9 @@ cudaError_t launch_plane_gemm(int64_t m, int64_t n, int64_t k_pad, const Oz2Modu
     um.kpart_steps = (um.ksteps + um.kparts - 1) / um.kparts;
     um.nunits *= um.kparts;
     if (um.kparts > 1) {
+      kern = plane_gemm_kernel<1, true>;  // same shared memory and threads, so the same pairs fit
+      err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+      if (err != cudaSuccess) return err;
       ctx.upart = reinterpret_cast<float*>(partials);
       ctx.ldu = magnitude_ldu(n);
       err = cudaMemsetAsync(ctx.upart, 0, static_cast<size_t>(m) * ctx.ldu * sizeof(float), st);
