@@ -142,7 +142,9 @@ __device__ __forceinline__ double crt_value(const int (&c)[R], int E, const Oz2M
   return round_to_double(top64, sticky, E, neg);
 }
 
-// Fast path: the same X by the direct CRT sum.  With u_k = c_k + coff_k ≥ 0,
+// The five-limb direct CRT (any r ≤ 16; the exact path tries it before
+// Garner for r ≥ 13): the same X by the direct CRT sum, kept exact over
+// six 32-bit limbs.  With u_k = c_k + coff_k ≥ 0,
 // S = Σ_k u_k W_k ≡ X (mod M), and S/M = Σ_k u_k y_k/m_k, so
 // q = ⌊S/M + 1/2⌋ gives X = S - q·M ∈ [-M/2, M/2).  q comes from the
 // 32.32 fixed-point sum Σ u_k F_k + 2^31, whose error is below
